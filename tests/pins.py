@@ -1,0 +1,348 @@
+"""Independent pins for the CPU oracle.
+
+Each ``check_*`` takes the oracle function(s) under test as arguments and
+raises AssertionError when they disagree with something the paper or plain
+mathematics fixes: a closed form, a library routine the special case reduces
+to, a brute-force enumeration, a hand-worked example or an invariant.  Tests
+call them with the real oracle (must pass) and with mutants that carry a
+planted mistake (must fail), which shows the pins can see such mistakes.
+"""
+from __future__ import annotations
+
+import itertools
+import math
+import os
+
+import numpy as np
+import torch
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _randn(g, *shape):
+    return g.standard_normal(shape)
+
+
+# ---------------------------------------------------------------- attention
+def check_single_key(cross_attn):
+    """kv_len = 1: softmax over one key has weight 1, so o = V[0] exactly."""
+    g = _rng(1)
+    B, H, D = 2, 3, 16
+    K = _randn(g, B, H, 4, D)
+    V = _randn(g, B, H, 4, D)
+    q = _randn(g, B, 1, H, D)
+    o = cross_attn(q, K, V, [1, 1])
+    assert np.array_equal(o[:, 0], V[:, :, 0, :]), "single key must return V[0]"
+
+
+def check_two_keys_closed_form(cross_attn):
+    """Two keys: o = sigma(s0 - s1) v0 + sigma(s1 - s0) v1 with s = q.k / sqrt(D)."""
+    g = _rng(2)
+    D = 8
+    for _ in range(5):
+        q = _randn(g, 1, 1, 1, D)
+        K = _randn(g, 1, 1, 2, D)
+        V = _randn(g, 1, 1, 2, D)
+        s0 = float(sum(q[0, 0, 0, d] * K[0, 0, 0, d] for d in range(D))) / math.sqrt(D)
+        s1 = float(sum(q[0, 0, 0, d] * K[0, 0, 1, d] for d in range(D))) / math.sqrt(D)
+        w0 = 1.0 / (1.0 + math.exp(s1 - s0))
+        want = w0 * V[0, 0, 0] + (1.0 - w0) * V[0, 0, 1]
+        got = cross_attn(q, K, V, [2])[0, 0, 0]
+        assert np.allclose(got, want, rtol=1e-13, atol=1e-13), "two-key closed form"
+
+
+def check_cross_vs_sdpa(cross_attn):
+    """Unmasked decode attention is torch's scaled_dot_product_attention (fp64)."""
+    g = _rng(3)
+    B, H, D, S = 2, 3, 32, 37
+    K = _randn(g, B, H, S + 5, D)
+    V = _randn(g, B, H, S + 5, D)
+    q = _randn(g, B, 1, H, D)
+    kv_len = [S, 11]
+    o = cross_attn(q, K, V, kv_len)
+    for b in range(B):
+        L = kv_len[b]
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[b].transpose(1, 0, 2)),          # [H, 1, D]
+            torch.from_numpy(K[b, :, :L]), torch.from_numpy(V[b, :, :L]))
+        assert np.allclose(o[b, 0], ref[:, 0].numpy(), rtol=1e-12, atol=1e-12), "cross vs SDPA"
+
+
+def check_chain_is_causal(tree_verify_attn):
+    """A chain tree is causal attention over prefix + chain (decode with a cache)."""
+    g = _rng(4)
+    B, H, D, n = 2, 2, 16, 6
+    kv_len = [9, 0]
+    K = _randn(g, B, H, 9 + n + 3, D)
+    V = _randn(g, B, H, 9 + n + 3, D)
+    q = _randn(g, B, n, H, D)
+    parent = np.stack([np.arange(-1, n - 1)] * B)
+    o = tree_verify_attn(q, parent, K, V, kv_len)
+    for b in range(B):
+        L = kv_len[b]
+        keep = torch.tensor([[k <= L + i for k in range(L + n)] for i in range(n)])
+        ref = torch.nn.functional.scaled_dot_product_attention(
+            torch.from_numpy(q[b].transpose(1, 0, 2)), torch.from_numpy(K[b, :, :L + n]),
+            torch.from_numpy(V[b, :, :L + n]), attn_mask=keep)
+        assert np.allclose(o[b], ref.numpy().transpose(1, 0, 2), rtol=1e-12, atol=1e-12), "chain != causal"
+
+
+def check_single_node_is_decode(tree_verify_attn):
+    """A one-node tree attends to the prefix plus its own key: plain decode over kv_len + 1 keys."""
+    g = _rng(5)
+    H, D, L = 3, 16, 20
+    K = _randn(g, 1, H, L + 4, D)
+    V = _randn(g, 1, H, L + 4, D)
+    q = _randn(g, 1, 1, H, D)
+    o = tree_verify_attn(q, np.array([[-1]]), K, V, [L])
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        torch.from_numpy(q[0].transpose(1, 0, 2)), torch.from_numpy(K[0, :, :L + 1]),
+        torch.from_numpy(V[0, :, :L + 1]))
+    assert np.allclose(o[0, 0], ref[:, 0].numpy(), rtol=1e-12, atol=1e-12), "single node != decode"
+
+
+def check_uniform_keys_mean(tree_verify_attn):
+    """Equal keys give equal scores, so o_i is the plain mean of V over the
+    keys query i may see: every prefix key plus its ancestors and itself.
+    Random V makes the mean identify exactly which rows were used."""
+    g = _rng(6)
+    H, D, L = 2, 8, 7
+    parent = np.array([-1, 0, 0, 1, 3, 2, 1, 4])
+    n = len(parent)
+    k = _randn(g, D)
+    K = np.broadcast_to(k, (1, H, L + n + 2, D)).copy()
+    V = _randn(g, 1, H, L + n + 2, D)
+    q = _randn(g, 1, n, H, D)
+    o = tree_verify_attn(q, parent[None], K, V, [L])
+    for i in range(n):
+        anc = set()
+        j = i
+        while j != -1:
+            anc.add(j)
+            j = parent[j]
+        rows = list(range(L)) + [L + j for j in sorted(anc)]
+        want = V[0][:, rows].mean(axis=1)
+        assert np.allclose(o[0, i], want, rtol=1e-12, atol=1e-12), f"uniform-key mean, node {i}"
+
+
+def check_planted_key(cross_attn):
+    """One key whose score exceeds every other by ~1000 takes all the weight:
+    o = V[k*] to within exp(-900).  Also needs a max-shifted softmax (exp(1000)
+    overflows fp64)."""
+    g = _rng(7)
+    D, L = 16, 50
+    K = _randn(g, 1, 1, L, D) * 0.01
+    q = _randn(g, 1, 1, 1, D)
+    kstar = 17
+    K[0, 0, kstar] = q[0, 0, 0] * (1000.0 * math.sqrt(D) / float(q[0, 0, 0] @ q[0, 0, 0]))
+    V = _randn(g, 1, 1, L, D)
+    o = cross_attn(q, K, V, [L])
+    assert np.all(np.isfinite(o)), "overflow in softmax"
+    assert np.allclose(o[0, 0, 0], V[0, 0, kstar], rtol=0, atol=1e-12), "planted key"
+
+
+def check_prefix_permutation(tree_verify_attn):
+    """Permuting the cached prefix rows (K and V together) leaves every output unchanged."""
+    g = _rng(8)
+    H, D, L = 2, 8, 13
+    parent = np.array([-1, 0, 1, 0])
+    n = len(parent)
+    K = _randn(g, 1, H, L + n, D)
+    V = _randn(g, 1, H, L + n, D)
+    q = _randn(g, 1, n, H, D)
+    o = tree_verify_attn(q, parent[None], K, V, [L])
+    perm = np.concatenate([g.permutation(L), np.arange(L, L + n)])
+    o2 = tree_verify_attn(q, parent[None], K[:, :, perm], V[:, :, perm], [L])
+    assert np.allclose(o, o2, rtol=1e-12, atol=1e-12), "prefix permutation"
+
+
+def check_tree_relabel(tree_verify_attn):
+    """Renumbering the tree nodes in another topological order (parents,
+    queries and tree K/V rows moved together) permutes the outputs likewise."""
+    g = _rng(9)
+    H, D, L = 2, 8, 5
+    parent = np.array([-1, 0, 0, 1, 1, 2, 3, 2])
+    n = len(parent)
+    K = _randn(g, 1, H, L + n, D)
+    V = _randn(g, 1, H, L + n, D)
+    q = _randn(g, 1, n, H, D)
+    o = tree_verify_attn(q, parent[None], K, V, [L])
+    # a different topological order: breadth-first with reversed sibling order
+    order = [0]
+    frontier = [0]
+    while frontier:
+        nxt = []
+        for p in frontier:
+            kids = [c for c in range(n) if parent[c] == p][::-1]
+            order += kids
+            nxt += kids
+        frontier = nxt
+    new_of = {old: new for new, old in enumerate(order)}
+    parent2 = np.array([-1 if parent[old] < 0 else new_of[parent[old]] for old in order])
+    rows = np.concatenate([np.arange(L), L + np.array(order)])
+    o2 = tree_verify_attn(q[:, order], parent2[None], K[:, :, rows], V[:, :, rows], [L])
+    assert np.allclose(o2, o[:, order], rtol=1e-12, atol=1e-12), "tree relabel"
+
+
+def read_cape_golden():
+    lines = [ln.strip() for ln in open(os.path.join(GOLDEN, "cape_mask_example.txt"))
+             if ln.strip() and not ln.startswith("#")]
+    gamma = int(lines[0].split()[1])
+    pos = [0] + [int(x) for x in lines[1].split()[1:]]
+    keep = np.array([[c == "1" for c in row] for row in lines[2:]])
+    return gamma, pos, keep
+
+
+def check_cape_mask_golden(cape_mask, tree_allowed_mask):
+    """The hand-worked CaPE mask example, from its equation and from the
+    ancestor rule on the equivalent tree (proposal spine + expansion leaves)."""
+    gamma, pos, keep = read_cape_golden()
+    assert np.array_equal(cape_mask(gamma, pos), keep), "CaPE mask vs hand-worked example"
+    parent = [-1] + [i - 1 for i in range(1, gamma + 1)] + [pos[i] - 1 for i in range(gamma + 1, len(pos))]
+    allowed = tree_allowed_mask(parent, 0)
+    assert allowed[:, 0].all(), "x_t must be visible to every tree token"
+    assert np.array_equal(allowed[1:, 1:], keep), "ancestor mask vs hand-worked CaPE mask"
+
+
+def check_cape_mask_random(cape_mask, tree_allowed_mask, cape_tree):
+    """On random CaPE shapes (S(p) in {7,5,3,1}, Section 3.2) the CaPE mask
+    equals the ancestor-or-self mask of the linearized tree."""
+    g = _rng(10)
+    for _ in range(50):
+        gamma = int(g.integers(1, 7))
+        sizes = [int(x) for x in g.choice([1, 3, 5, 7], size=gamma)]
+        parent, pos = cape_tree(sizes)
+        allowed = tree_allowed_mask(parent, 0)
+        assert np.array_equal(allowed[1:, 1:], cape_mask(gamma, pos)), "CaPE mask != ancestor mask"
+
+
+# ---------------------------------------------------------------- acceptance
+def read_accept_golden():
+    ex, cur = [], None
+    for ln in open(os.path.join(GOLDEN, "accept_examples.txt")):
+        ln = ln.strip()
+        if not ln or ln.startswith("#"):
+            continue
+        key, *vals = ln.split()
+        if key == "example":
+            cur = {"name": vals[0]}
+            ex.append(cur)
+        else:
+            cur[key] = [int(v) for v in vals]
+    return ex
+
+
+def logits_with_argmax(argmax, vocab, g):
+    lg = g.standard_normal((len(argmax), vocab)).astype(np.float32)
+    for i, a in enumerate(argmax):
+        lg[i, a] = lg[i].max() + 1.0
+    return lg
+
+
+def check_accept_golden(tree_accept):
+    g = _rng(11)
+    for ex in read_accept_golden():
+        n = len(ex["parent"])
+        lg = logits_with_argmax(ex["argmax"], 16, g)[None]
+        path, ln, bonus = tree_accept(np.array([ex["draft"]]), np.array([ex["parent"]]), lg)
+        want = ex["path"] + [-1] * (n - len(ex["path"]))
+        assert list(path[0]) == want, ex["name"]
+        assert int(ln[0]) == ex["len"][0] and int(bonus[0]) == ex["bonus"][0], ex["name"]
+
+
+def brute_force_accept(draft, parent, argmax):
+    """Enumerate every root-to-node path and keep the longest fully matching
+    one (ties: the path ending at the lowest node index)."""
+    n = len(parent)
+    best = (0, 0)
+    for c in range(n):
+        chain = [c]
+        while chain[-1] != 0:
+            chain.append(int(parent[chain[-1]]))
+        chain.reverse()
+        if all(int(draft[chain[k + 1]]) == int(argmax[chain[k]]) for k in range(len(chain) - 1)):
+            if (len(chain) - 1, -c) > (best[0], -best[1]):
+                best = (len(chain) - 1, c)
+    d, c = best
+    chain = [c]
+    while chain[-1] != 0:
+        chain.append(int(parent[chain[-1]]))
+    return chain[::-1], d, int(argmax[c])
+
+
+def random_small_tree(g, n):
+    return np.array([-1] + [int(g.integers(i)) for i in range(1, n)])
+
+
+def check_accept_brute_force(tree_accept):
+    g = _rng(12)
+    for trial in range(300):
+        n = int(g.integers(1, 13))
+        vocab = int(g.integers(2, 5))          # tiny vocab: many matches and ties
+        parent = random_small_tree(g, n)
+        draft = g.integers(vocab, size=n)
+        lg = g.integers(-2, 3, size=(n, vocab)).astype(np.float32)   # integer logits: frequent ties
+        argmax = [min(v for v in range(vocab) if lg[i, v] == lg[i].max()) for i in range(n)]
+        chain, d, bonus = brute_force_accept(draft, parent, argmax)
+        path, ln, bo = tree_accept(draft[None], parent[None], lg[None])
+        assert list(path[0][:d + 1]) == chain and all(path[0][d + 1:] == -1), f"trial {trial}"
+        assert int(ln[0]) == d and int(bo[0]) == bonus, f"trial {trial}"
+
+
+def check_accept_chain_is_sd(tree_accept):
+    """On a chain, acceptance is plain SD: the longest matching prefix of the
+    proposal, then the target's token after it (Section 2)."""
+    g = _rng(13)
+    for _ in range(100):
+        n = int(g.integers(1, 10))
+        vocab = 3
+        draft = g.integers(vocab, size=n)
+        lg = g.standard_normal((n, vocab)).astype(np.float32)
+        a = [int(np.argmax(lg[i])) for i in range(n)]
+        k = 0
+        while k + 1 < n and draft[k + 1] == a[k]:
+            k += 1
+        path, ln, bo = tree_accept(draft[None], np.arange(-1, n - 1)[None], lg[None])
+        assert int(ln[0]) == k and int(bo[0]) == a[k] and list(path[0][:k + 1]) == list(range(k + 1))
+
+
+def check_accept_greedy_equivalence(tree_accept):
+    """With distinct sibling tokens the kept tokens plus the bonus are exactly
+    what greedy decoding with the target emits while the tree can follow it."""
+    g = _rng(14)
+    for _ in range(200):
+        n = int(g.integers(2, 16))
+        vocab = 16                               # > n, so siblings can always be distinct
+        parent = random_small_tree(g, n)
+        draft = np.zeros(n, dtype=np.int64)
+        for p in range(n):
+            kids = [c for c in range(n) if parent[c] == p]
+            if kids:
+                draft[kids] = g.choice(vocab, size=len(kids), replace=False)
+        lg = (g.standard_normal((n, vocab)) * 0.1).astype(np.float32)
+        for p in range(n):                       # make the target follow the tree often
+            kids = [c for c in range(n) if parent[c] == p]
+            if kids and g.random() < 0.7:
+                lg[p, draft[kids[int(g.integers(len(kids)))]]] = 5.0
+        a = np.argmax(lg, axis=1)
+        node, emitted = 0, []
+        while True:
+            nxt = [c for c in range(n) if parent[c] == node and draft[c] == a[node]]
+            if not nxt:
+                emitted.append(int(a[node]))
+                break
+            node = nxt[0]
+            emitted.append(int(draft[node]))
+        path, ln, bo = tree_accept(draft[None], parent[None], lg[None])
+        got = [int(draft[c]) for c in path[0][1:int(ln[0]) + 1]] + [int(bo[0])]
+        assert got == emitted
+
+
+def check_argmax_ties(row_argmax):
+    lg = np.array([[1.0, 3.0, 3.0, 2.0], [5.0, 5.0, 5.0, 5.0], [-1.0, -2.0, -1.0, -3.0],
+                   [0.0, -0.0, 0.0, -1.0]], dtype=np.float32)
+    assert list(row_argmax(lg)) == [1, 0, 0, 0]
