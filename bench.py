@@ -1,0 +1,457 @@
+"""Benchmark of one GliDe-with-CaPE speculative round on the KV cache.
+
+One step = the whole hot path for one target layer on one batch:
+gamma = 5 sequential glide_cross_attn calls (draft steps), one tree_verify_attn
+over the expanded proposal tree, one tree_accept.  Default workload: the
+Vicuna-33B-shaped long-context case (B=4, H=52, D=128, kv_len=16384, bf16,
+64-node trees), whose K/V (1.75 GB) is far larger than L2, so no flush is
+needed between steps.
+
+Prints ONE JSON line.  `value` is the KV-cache bytes the step reads
+(gamma cross-attention passes + one verification pass) divided by the device
+time of the step.  --impl reference times the fp64 CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2402_02082_gb300 import synth  # noqa: E402
+
+METRIC = "KV-cache HBM GB/s and fraction of ~8 TB/s peak; verified tree tokens/sec per layer"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ------------------------------------------------------------------ helpers
+def kv_bytes(w: synth.Workload):
+    """Algorithmic bytes: (cross per call, verify per call) of K/V reads only."""
+    e = 2 if w.dtype == "bf16" else 4
+    cross = sum(w.H * L * w.D * 2 * e for L in w.kv_len)
+    verify = sum(w.H * (L + w.n) * w.D * 2 * e for L in w.kv_len)
+    return cross, verify
+
+
+def algo_bytes(w: synth.Workload):
+    """Algorithmic bytes per launch of each kernel, inputs read + outputs written."""
+    e = 2 if w.dtype == "bf16" else 4
+    cross_kv, verify_kv = kv_bytes(w)
+    cross = cross_kv + w.B * w.H * w.D * (e + 4) + 4 * w.B
+    verify = verify_kv + w.B * w.n * w.H * w.D * (e + 4) + 4 * w.B * (w.n + 1)
+    accept = w.B * w.n * (w.vocab * 4 + 4 + 4 + 4) + 8 * w.B
+    return {"glide_cross_attn": cross, "tree_verify_attn": verify, "tree_accept": accept}
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash(fname):
+    p = os.path.join(ROOT, "paper_2402_02082_gb300", "csrc", fname)
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+KERNEL_FILES = {"glide_cross_attn": "cross_attn.cu", "tree_verify_attn": "tree_attn_tc.cu",
+                "tree_accept": "accept.cu"}
+
+
+def recorded_traffic(kernel, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current source of that kernel; else None."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    rec = d.get(kernel, {}).get(workload)
+    if not rec or rec.get("source_sha256_16") != kernel_source_hash(KERNEL_FILES[kernel]):
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------- CPU oracle baseline
+def _oracle_pair(args):
+    """Oracle for one (b, h) of the step: gamma cross-attention calls + the
+    tree verification (one slab of K/V)."""
+    import oracle
+    q_draft, q_tree, parent, Kbh, Vbh, L = args
+    t0 = time.perf_counter()
+    for i in range(q_draft.shape[0]):
+        oracle.cross_attn(q_draft[i][None, None, None, :], Kbh[None, None], Vbh[None, None], [L])
+    oracle.tree_verify_attn(q_tree[None, :, None, :], parent[None], Kbh[None, None], Vbh[None, None], [L])
+    return time.perf_counter() - t0
+
+
+def oracle_sample_args(w, case, pairs):
+    out = []
+    for b, h in pairs:
+        L = w.kv_len[b]
+        out.append((case["q_draft"][:, b, 0, h, :], case["q_tree"][b, :, h, :], case["parent_idx"][b],
+                    np.ascontiguousarray(case["K"][b, h, :L + w.n]), np.ascontiguousarray(case["V"][b, h, :L + w.n]),
+                    L))
+    return out
+
+
+def time_oracle(w, case, pairs, pool, cores):
+    """KV GB/s of the oracle over `pairs` (b, h) slabs, with `cores` single-threaded workers."""
+    args = oracle_sample_args(w, case, pairs)
+    e = 2 if w.dtype == "bf16" else 4
+    t0 = time.perf_counter()
+    pool.map(_oracle_pair, args, chunksize=1)
+    dt = time.perf_counter() - t0
+    nbytes = sum(w.gamma * w.kv_len[b] * w.D * 2 * e + (w.kv_len[b] + w.n) * w.D * 2 * e for b, _ in pairs)
+    return nbytes / dt / 1e9, dt
+
+
+def make_pool(cores):
+    os.environ["OMP_NUM_THREADS"] = "1"
+    os.environ["OPENBLAS_NUM_THREADS"] = "1"
+    os.environ["MKL_NUM_THREADS"] = "1"
+    return mp.get_context("spawn").Pool(cores)
+
+
+def pick_pairs(w, k, seed):
+    g = np.random.default_rng(seed)
+    allp = [(b, h) for b in range(w.B) for h in range(w.H)]
+    idx = g.choice(len(allp), size=min(k, len(allp)), replace=False)
+    return [allp[i] for i in sorted(idx)]
+
+
+# --------------------------------------------------------------- reference
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    w = synth.workload(args.workload)
+    case = synth.make_case(w, garbage="zero")
+    cores = os.cpu_count() or 1
+    pool = make_pool(cores)
+    per_step = max(1, min(w.B * w.H, cores))
+    for s in range(args.warmup):
+        time_oracle(w, case, pick_pairs(w, per_step, 10_000 + s), pool, cores)
+    total_bytes, total_t = 0.0, 0.0
+    e = 2 if w.dtype == "bf16" else 4
+    for s in range(args.steps):
+        pairs = pick_pairs(w, per_step, s)
+        gbs, dt = time_oracle(w, case, pairs, pool, cores)
+        total_t += dt
+        total_bytes += gbs * dt * 1e9
+    pool.close()
+    value = total_bytes / total_t / 1e9
+    sample = (f"{per_step} of {w.B * w.H} (b,h) slabs per step: gamma={w.gamma} cross-attention calls + "
+              f"tree verification each, fp64 numpy oracle, {cores} single-threaded worker processes")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total_t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(w),
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def workload_config(w):
+    return {"workload": w.name, "B": w.B, "H": w.H, "D": w.D, "kv_len": list(w.kv_len) if w.B <= 8 else "ragged",
+            "tree_nodes": w.n, "gamma": w.gamma, "vocab": w.vocab, "dtype": w.dtype,
+            "l2": "inputs larger than L2 (no flush)" if sum(kv_bytes(w)) > 2 * 129e6 else "L2 flushed between steps"}
+
+
+# -------------------------------------------------------------------- main
+def run_glide(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2402_02082_gb300 import binding as gb
+    from paper_2402_02082_gb300 import build
+
+    if rank == 0 or world == 1:
+        build.build()
+    if world > 1:
+        dist.barrier()
+    build.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = synth.workload(args.workload)
+
+    cpu = None
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        pool = make_pool(cores)   # spawned before any GPU work
+        cpu = (pool, cores)
+
+    case = synth.make_case(w, garbage="zero")
+
+    def to_dev(a):
+        if a.dtype == np.uint16:
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+    K, V = to_dev(case["K"]), to_dev(case["V"])
+    q_draft = [to_dev(case["q_draft"][i]) for i in range(w.gamma)]
+    q_tree = to_dev(case["q_tree"])
+    parent = to_dev(case["parent_idx"].astype(np.int32))
+    kv_len = to_dev(np.asarray(w.kv_len, dtype=np.int32))
+    draft = to_dev(case["draft_tokens"].astype(np.int32))
+    logits = to_dev(case["target_logits"])
+    B, H, S_cap, D = case["K"].shape
+    n = w.n
+    desc = gb.make_desc(B, H, D, S_cap, gb.GLIDE_BF16 if w.dtype == "bf16" else gb.GLIDE_F32)
+    ws = torch.zeros(gb.glide_attn_workspace_bytes(desc, n), dtype=torch.uint8, device=dev)
+    ws_acc = torch.zeros(gb.glide_accept_workspace_bytes(B, n), dtype=torch.uint8, device=dev)
+    out_c = [torch.empty(B, 1, H, D, device=dev) for _ in range(w.gamma)]
+    out_t = torch.empty(B, n, H, D, device=dev)
+    path = torch.empty(B, n, dtype=torch.int32, device=dev)
+    ln = torch.empty(B, dtype=torch.int32, device=dev)
+    bonus = torch.empty(B, dtype=torch.int32, device=dev)
+    flags = gb.GLIDE_FLAG_FORCE_FMA if args.force_fma else 0
+
+    names = ["glide_cross_attn"] * w.gamma + ["tree_verify_attn", "tree_accept"]
+
+    def launches():
+        for i in range(w.gamma):
+            yield lambda i=i: gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws)
+        yield lambda: gb.tree_verify_attn(q_tree, parent, K, V, kv_len, w.max_kv_len, out_t, ws, flags=flags)
+        yield lambda: gb.tree_accept(draft, parent, logits, path, ln, bonus, ws_acc)
+
+    step_fns = list(launches())
+    stream = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        for f in step_fns:
+            f()
+    torch.cuda.synchronize()
+    if gb.glide_read_device_status(ws) != gb.GLIDE_OK or gb.glide_read_device_status(ws_acc) != gb.GLIDE_OK:
+        raise RuntimeError("device status not OK after warm-up")
+
+    # ---- device-timed region: inputs resident in HBM
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in step_fns]
+          for _ in range(args.steps)]
+    t_begin, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local_rank)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    t_begin.record(stream)
+    for s in range(args.steps):
+        for j, f in enumerate(step_fns):
+            ev[s][j][0].record(stream)
+            f()
+            ev[s][j][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = t_begin.elapsed_time(t_end)
+    per_kernel = {}
+    for j, nm in enumerate(names):
+        per_kernel.setdefault(nm, []).extend(ev[s][j][0].elapsed_time(ev[s][j][1]) for s in range(args.steps))
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    if gb.glide_read_device_status(ws) != gb.GLIDE_OK or gb.glide_read_device_status(ws_acc) != gb.GLIDE_OK:
+        raise RuntimeError("device status not OK after the timed region")
+
+    cross_kv, verify_kv = kv_bytes(w)
+    step_kv = w.gamma * cross_kv + verify_kv
+    value = world * step_kv * args.steps / (elapsed_ms * 1e-3) / 1e9
+    tree_tok = world * B * n * args.steps / (elapsed_ms * 1e-3)
+
+    # ---- end to end: per-round inputs from pinned host memory, results back to host
+    e2e_steps = max(3, min(args.steps, args.e2e_steps))
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    h_qd = [pin(case["q_draft"][i].view(np.int16)) for i in range(w.gamma)]
+    h_qt = pin(case["q_tree"].view(np.int16) if case["q_tree"].dtype == np.uint16 else case["q_tree"])
+    h_par = pin(case["parent_idx"].astype(np.int32))
+    h_kv = pin(np.asarray(w.kv_len, dtype=np.int32))
+    h_dr = pin(case["draft_tokens"].astype(np.int32))
+    h_lg = pin(case["target_logits"])
+    tk = [pin(case["K"][b, :, w.kv_len[b]:w.kv_len[b] + n].view(np.int16)) for b in range(B)]
+    tv = [pin(case["V"][b, :, w.kv_len[b]:w.kv_len[b] + n].view(np.int16)) for b in range(B)]
+    r_c = [torch.empty(B, 1, H, D).pin_memory() for _ in range(w.gamma)]
+    r_t = torch.empty(B, n, H, D).pin_memory()
+    r_p = torch.empty(B, n, dtype=torch.int32).pin_memory()
+    r_l = torch.empty(B, dtype=torch.int32).pin_memory()
+    r_b = torch.empty(B, dtype=torch.int32).pin_memory()
+    K16, V16 = K.view(torch.int16), V.view(torch.int16)
+
+    def e2e_step():
+        kv_len.copy_(h_kv, non_blocking=True)
+        for b in range(B):
+            K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tk[b], non_blocking=True)
+            V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tv[b], non_blocking=True)
+        for i in range(w.gamma):
+            q_draft[i].view(torch.int16).copy_(h_qd[i], non_blocking=True)
+            gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws)
+            r_c[i].copy_(out_c[i], non_blocking=True)
+        q_tree.view(torch.int16).copy_(h_qt, non_blocking=True)
+        parent.copy_(h_par, non_blocking=True)
+        gb.tree_verify_attn(q_tree, parent, K, V, kv_len, w.max_kv_len, out_t, ws, flags=flags)
+        r_t.copy_(out_t, non_blocking=True)
+        draft.copy_(h_dr, non_blocking=True)
+        logits.copy_(h_lg, non_blocking=True)
+        gb.tree_accept(draft, parent, logits, path, ln, bonus, ws_acc)
+        r_p.copy_(path, non_blocking=True)
+        r_l.copy_(ln, non_blocking=True)
+        r_b.copy_(bonus, non_blocking=True)
+        torch.cuda.synchronize()
+
+    h2d = (sum(t.numel() * t.element_size() for t in h_qd) + h_qt.numel() * h_qt.element_size() +
+           h_par.numel() * 4 + h_kv.numel() * 4 + h_dr.numel() * 4 + h_lg.numel() * 4 +
+           sum(t.numel() * 2 for t in tk) + sum(t.numel() * 2 for t in tv))
+    d2h = sum(t.numel() * 4 for t in r_c) + r_t.numel() * 4 + r_p.numel() * 4 + 8 * B
+    for _ in range(2):
+        e2e_step()
+    if world > 1:
+        dist.barrier()
+    e0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    e2e_s = time.perf_counter() - e0
+    if world > 1:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e_value = world * step_kv * e2e_steps / e2e_s / 1e9
+
+    # ---- roofline of the dominant kernel
+    peak, peak_src = measured_peaks()
+    ab = algo_bytes(w)
+    kernels = {}
+    for nm, times in per_kernel.items():
+        avg_ms = sum(times) / len(times)
+        ach = ab[nm] / (avg_ms * 1e-3) / 1e9
+        kernels[nm] = {"avg_us": 1e3 * avg_ms, "launches_per_step": names.count(nm),
+                       "share": names.count(nm) * avg_ms * args.steps / sum(sum(v) for v in per_kernel.values()),
+                       "algo_bytes_per_launch": ab[nm], "achieved_gbs": ach, "frac_of_peak": ach / peak}
+    dom = max(kernels, key=lambda k: kernels[k]["share"])
+    roof = {"kernel": dom, "bound": "hbm", "achieved": kernels[dom]["achieved_gbs"], "peak": peak,
+            "peak_source": peak_src, "unit": "GB/s", "frac": kernels[dom]["frac_of_peak"],
+            "traffic": recorded_traffic(dom, w.name)}
+
+    cpu_baseline = None
+    if cpu is not None:
+        pool, cores = cpu
+        pairs = pick_pairs(w, args.cpu_pairs, 1234)
+        gbs, dt = time_oracle(w, case, pairs, pool, cores)
+        pool.close()
+        cpu_baseline = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                        "sample": f"{len(pairs)} of {B * H} (b,h) slabs: gamma={w.gamma} cross-attention calls + "
+                                  f"tree verification each; fp64 numpy oracle, {cores} single-threaded workers, "
+                                  f"{dt:.1f} s wall"}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+                "config": workload_config(w),
+                "frac_of_nominal_8tbs": value / world / NOMINAL_HBM_GBS,
+                "frac_of_measured_hbm": value / world / peak,
+                "tree_tokens_per_s_per_layer": tree_tok,
+                "roofline": roof, "kernels": kernels, "cpu_baseline": cpu_baseline,
+                "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                        "steps": e2e_steps},
+                "gpu_launches": len(step_fns) * args.steps, "clocks": clk}
+        if args.force_fma:
+            line["config"]["tree_kernel"] = "cuda-core (forced)"
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["glide", "reference"], default="glide")
+    ap.add_argument("--workload", default="vicuna33b-long-b4", choices=[w.name for w in synth.workloads()])
+    ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--cpu-pairs", type=int, default=64)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--force-fma", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    return run_glide(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

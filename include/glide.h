@@ -1,0 +1,175 @@
+/*
+ * glide.h -- C ABI of libglide: the KV-cache attention hot path of
+ * GliDe-with-CaPE speculative decoding (arXiv 2402.02082) on GB300 (sm_103a).
+ *
+ * Three calls make up one speculative round for one target layer:
+ *
+ *   glide_cross_attn   the GliDe draft model's cross-attention: a draft query
+ *                      per (sequence, head) attends to every cached key/value
+ *                      of the frozen target model (Section 3.1, the hd_j
+ *                      equation; no mask at inference).
+ *   tree_verify_attn   the target's parallel verification of the linearized
+ *                      expanded proposal: n tree queries attend to the cached
+ *                      prefix and to their own ancestors and themselves
+ *                      (the CaPE mask of Section 3.2 is this mask on CaPE's
+ *                      trees).
+ *   tree_accept        greedy acceptance on the token tree (Section 2): the
+ *                      deepest node whose whole root path the target's argmax
+ *                      reproduces, and the free bonus token.
+ *
+ * Conventions shared by all calls
+ * -------------------------------
+ * - Every tensor pointer is a DEVICE pointer owned by the caller; the library
+ *   allocates nothing and keeps no state between calls.  All work is enqueued
+ *   on `stream` (a cudaStream_t; NULL means the legacy default stream) and is
+ *   asynchronous: a returned GLIDE_OK means "launched", not "finished".
+ * - Layouts are dense, row-major, no padding:
+ *     queries   [B, nq, H, D]          (nq = 1 for cross-attention, n for the tree)
+ *     K, V      [B, H, S_cap, D]       one contiguous S_cap x D slab per (b, h)
+ *     out       [B, nq, H, D] fp32
+ *     kv_len    [B] int32              cached prefix length of each sequence
+ *     parent    [B, n] int32           linearized tree: -1 for a root, else an
+ *                                      earlier node (parent[i] < i)
+ * - The tree's own keys/values must already be written at cache rows
+ *   kv_len[b] .. kv_len[b]+n-1, in linearized order (node j at row kv_len[b]+j).
+ *   Rows at and beyond kv_len[b]+n are never read and may hold anything.
+ * - Rotary embedding (if any) is applied by the caller before the call.
+ * - Host-side checks run before anything is launched; a bad argument returns
+ *   GLIDE_ERR_INVALID and touches no memory.  Device-resident values
+ *   (kv_len, parent, draft tokens) cannot be checked on the host: the kernels
+ *   clamp them into range, so bad values give meaningless results but never an
+ *   out-of-bounds access.
+ * - Workspace: caller-allocated device memory of at least the size the
+ *   matching *_workspace_bytes function returns, ZERO-FILLED before its first
+ *   use.  It holds a status word, arrival counters (and, for tree_accept,
+ *   argmax slots) that must start at zero, and scratch for split partial
+ *   results.  Every successful call returns the words that must start at zero
+ *   to zero, so one buffer can be reused across calls on the same stream.
+ *   Calls that run concurrently on different streams need separate
+ *   workspaces.
+ * - Kernel waits are bounded.  A kernel that gives up waiting records
+ *   GLIDE_ERR_DEVICE_TIMEOUT in its workspace; glide_read_device_status reads
+ *   and clears it.
+ */
+#ifndef GLIDE_H
+#define GLIDE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GLIDE_ABI_VERSION 1
+
+typedef struct CUstream_st* glide_stream_t;
+
+typedef enum {
+  GLIDE_OK = 0,
+  GLIDE_ERR_INVALID = 1,        /* bad argument found on the host; nothing launched        */
+  GLIDE_ERR_UNSUPPORTED = 2,    /* well-formed but outside the supported shapes            */
+  GLIDE_ERR_CUDA = 3,           /* a CUDA runtime call or kernel launch failed             */
+  GLIDE_ERR_DEVICE_TIMEOUT = 4  /* a kernel gave up a bounded wait (device status only)    */
+} glide_status;
+
+typedef enum { GLIDE_BF16 = 0, GLIDE_F32 = 1 } glide_dtype;
+
+/* flags */
+#define GLIDE_FLAG_FORCE_FMA 1u   /* tree_verify_attn: use the CUDA-core kernel even where the
+                                     tensor-core kernel applies (testing and comparison)     */
+
+typedef struct {
+  int32_t B;          /* sequences in the batch, 1..1024                                   */
+  int32_t H;          /* attention heads (of the target layer), >= 1                       */
+  int32_t D;          /* head dimension d_k: 64 or 128                                     */
+  int32_t S_cap;      /* rows of each (b, h) slab of the K/V cache                          */
+  glide_dtype dtype;  /* element type of queries, K and V                                   */
+  float scale;        /* softmax scale; 0 means 1/sqrt(D) (Section 3.1)                     */
+  uint32_t flags;     /* GLIDE_FLAG_* bits                                                  */
+  int32_t max_ctas;   /* upper bound on the CTAs of one attention launch; 0 = automatic     */
+} glide_attn_desc;
+
+/* Version of this ABI (GLIDE_ABI_VERSION of the built library). */
+int32_t glide_abi_version(void);
+
+/* Static, human-readable name of a status code. */
+const char* glide_status_str(glide_status status);
+
+/* Bytes of workspace that glide_cross_attn (n_queries = 1) and
+ * tree_verify_attn (n_queries = n) need for this descriptor; 0 if the
+ * descriptor is invalid.  A buffer sized for the largest n serves both. */
+size_t glide_attn_workspace_bytes(const glide_attn_desc* desc, int32_t n_queries);
+
+/* Bytes of workspace that tree_accept needs for B trees of n nodes. */
+size_t glide_accept_workspace_bytes(int32_t B, int32_t n);
+
+/*
+ * GliDe cross-attention (Section 3.1):
+ *   out[b,0,h,:] = SoftMax(q[b,0,h,:] . K[b,h,k,:] * scale, k < kv_len[b]) V[b,h,k,:]
+ * q_draft [B,1,H,D] (desc->dtype), K_cache/V_cache [B,H,S_cap,D] (desc->dtype),
+ * kv_len [B] int32 on the device, clamped to [0, max_kv_len]; a sequence with
+ * kv_len 0 has nothing to attend to and gets zeros.
+ * max_kv_len: host-side upper bound of kv_len, 1 <= max_kv_len <= S_cap.
+ * out [B,1,H,D] fp32.
+ */
+glide_status glide_cross_attn(const glide_attn_desc* desc, const void* q_draft,
+                              const void* K_cache, const void* V_cache,
+                              const int32_t* kv_len, int32_t max_kv_len, float* out,
+                              void* workspace, size_t workspace_bytes, glide_stream_t stream);
+
+/*
+ * Tree verification attention (Section 3.2, CaPE verification mask; the
+ * ancestor-or-self rule of the token-tree verifier it borrows):
+ *   out[b,i,h,:] = SoftMax over k in A_i of (q[b,i,h,:] . K[b,h,k,:] * scale) V[b,h,k,:]
+ *   A_i = {0 .. kv_len[b]-1} U {kv_len[b] + j : j = i or j an ancestor of i}
+ * q_tree [B,n,H,D], 1 <= n <= 64; parent_idx [B,n] int32 on the device (a forest
+ * in topological order; an entry outside [-1, i) is treated as -1).
+ * kv_len [B] on the device, clamped to [0, max_kv_len]; 0 <= max_kv_len and
+ * max_kv_len + n <= S_cap.  out [B,n,H,D] fp32.
+ */
+glide_status tree_verify_attn(const glide_attn_desc* desc, const void* q_tree, int32_t n,
+                              const int32_t* parent_idx, const void* K_cache,
+                              const void* V_cache, const int32_t* kv_len, int32_t max_kv_len,
+                              float* out, void* workspace, size_t workspace_bytes,
+                              glide_stream_t stream);
+
+/*
+ * Greedy tree acceptance (Section 2, greedy "speculative decoding" rule, on
+ * the token tree of Section 3.2):
+ *   a_i  = argmax_v target_logits[b,i,v] (lowest v among equal maxima; -0 == +0)
+ *   node c >= 1 with parent p is accepted iff draft_tokens[b,c] == a_p and p is
+ *   accepted; node 0 (x_t, the last accepted token) is always accepted.
+ *   Result: the accepted node of greatest depth (lowest index among equals).
+ * draft_tokens [B,n] int32, parent_idx [B,n] int32 (node 0 the root, every other
+ * parent earlier; an entry outside [0, i) makes node i unreachable),
+ * target_logits [B,n,V] fp32, finite.  1 <= n <= 64, 1 <= V.
+ * Outputs: path [B,n] int32 = root..node node indices, -1 padded;
+ * len [B] int32 = depth of that node (accepted proposal tokens);
+ * bonus [B] int32 = a_node, the target's free next token.
+ */
+glide_status tree_accept(const int32_t* draft_tokens, const int32_t* parent_idx,
+                         const float* target_logits, int32_t B, int32_t n, int32_t V,
+                         int32_t* path, int32_t* len, int32_t* bonus,
+                         void* workspace, size_t workspace_bytes, glide_stream_t stream);
+
+/*
+ * Host-side check of a parent array (HOST memory, [B,n]): every entry is -1 or
+ * in [0, i).  With require_root0 != 0 (the tree_accept convention) node 0 must
+ * be the only root.  Returns GLIDE_OK or GLIDE_ERR_INVALID.
+ */
+glide_status glide_validate_tree(const int32_t* parent_idx_host, int32_t B, int32_t n,
+                                 int32_t require_root0);
+
+/*
+ * Waits for `stream`, then returns the status the kernels recorded in
+ * `workspace` (GLIDE_OK or GLIDE_ERR_DEVICE_TIMEOUT) and clears it.  Works on
+ * attention and acceptance workspaces alike.
+ */
+glide_status glide_read_device_status(void* workspace, glide_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GLIDE_H */

@@ -1,0 +1,221 @@
+// Device-side building blocks shared by the attention and acceptance kernels:
+// mbarrier and bulk-copy wrappers with bounded waits, the split-KV work
+// partition over all (sequence, head) key ranges, and the log-sum-exp merge
+// of partial softmax results.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace glide {
+
+constexpr uint32_t kStatusTimeout = 4;          // GLIDE_ERR_DEVICE_TIMEOUT
+constexpr uint64_t kWaitLimitNs = 1000000000ull; // 1 s: far beyond any legitimate wait
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ---------------------------------------------------------------- workspace
+// Attention workspace: [0,256) status word; [256, 256 + 4*B*H) per-(b,h)
+// arrival counters; then 256-aligned partial slots of nq*(D+2) floats.
+struct WsLayout {
+  static constexpr size_t kHeader = 256;
+  static __host__ __device__ size_t counters_off() { return kHeader; }
+  static __host__ __device__ size_t partials_off(int B, int H) {
+    size_t c = kHeader + sizeof(unsigned) * (size_t)B * H;
+    return (c + 255) & ~size_t(255);
+  }
+};
+
+// -------------------------------------------------------------------- misc
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void record_status(unsigned* status, unsigned code) {
+  atomicCAS(status, 0u, code);
+}
+
+// bf16 pair (one 32-bit word, element 0 in the low half) -> two floats.
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// ---------------------------------------------------------------- mbarrier
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Waits for the phase of `bar` with the given parity to complete.  Gives up
+// after kWaitLimitNs, or at once when another thread of the CTA has set
+// *abort; on giving up it records the timeout, sets *abort and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          unsigned* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      *abort = 1;
+      record_status(status, kStatusTimeout);
+      return false;
+    }
+  }
+}
+
+// ------------------------------------------------------------- bulk copies
+// 1-D bulk copy global -> this CTA's shared memory, completing `bytes` of
+// transaction count on `bar`.  dst, src and bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
+                                         uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// Named barrier among the `nthreads` consumer threads (id 1; id 0 is __syncthreads).
+__device__ __forceinline__ void consumer_sync(int nthreads) {
+  asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
+}
+
+// --------------------------------------------------------------- partition
+// Every (b, h) owns a run of `ntiles(b)` consecutive tiles in one global
+// sequence (b-major, then h, then key tile).  The G CTAs of a launch take
+// equal contiguous shares of that sequence (sizes differ by at most one), so
+// ragged batches stay balanced.  A CTA's share is cut into segments at (b, h)
+// boundaries.  Tiles cover keys [t*TK, t*TK + TK) of a slab.
+struct Partition {
+  long long total;
+  long long base;
+  long long rem;
+  int G;
+  __device__ void init(long long total_tiles, int grid) {
+    total = total_tiles;
+    G = grid;
+    base = total / grid;
+    rem = total % grid;
+  }
+  __device__ long long begin(int c) const { return (long long)c * base + (c < rem ? c : rem); }
+  __device__ long long end(int c) const { return begin(c) + base + (c < rem ? 1 : 0); }
+  __device__ int cta_of(long long g) const {
+    const long long big = rem * (base + 1);
+    if (g < big) return (int)(g / (base + 1));
+    return (int)(rem + (g - big) / base);
+  }
+};
+
+// Per-sequence tile bookkeeping kept in shared memory.
+struct BatchTiles {
+  long long* start;  // [B+1]: first global tile of sequence b (over all its heads)
+  int* len;          // [B]  : keys attended per slab (prefix, plus tree nodes)
+  int* ntiles;       // [B]  : tiles per (b, h)
+  int* plen;         // [B]  : clamped prefix length kv_len[b]
+};
+
+// Fills BatchTiles (all threads of the block must call; ends with __syncthreads).
+// keys(b) = clamp(kv_len[b], 0, max_kv_len) + extra.
+__device__ inline void build_batch_tiles(BatchTiles bt, const int* kv_len, int B, int H,
+                                         int max_kv_len, int extra, int TK) {
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    int L = kv_len[b];
+    L = L < 0 ? 0 : (L > max_kv_len ? max_kv_len : L);
+    bt.plen[b] = L;
+    bt.len[b] = L + extra;
+    bt.ntiles[b] = (L + extra + TK - 1) / TK;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long s = 0;
+    for (int b = 0; b < B; ++b) {
+      bt.start[b] = s;
+      s += (long long)H * bt.ntiles[b];
+    }
+    bt.start[B] = s;
+  }
+  __syncthreads();
+}
+
+struct Segment {
+  int b, h;
+  int t0, t1;          // tile range within the (b, h) slab, [t0, t1)
+  long long g_end;     // global index one past the segment
+  int c_first, c_last; // CTAs that share this (b, h)
+};
+
+// Locates the segment that starts at global tile g (< g_limit, the CTA's end).
+__device__ inline Segment locate(const BatchTiles& bt, const Partition& P, int B, long long g,
+                                 long long g_limit) {
+  int lo = 0, hi = B - 1;  // last b with start[b] <= g
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (bt.start[mid] <= g) lo = mid; else hi = mid - 1;
+  }
+  Segment s;
+  s.b = lo;
+  const int nt = bt.ntiles[lo];
+  const long long off = g - bt.start[lo];
+  s.h = (int)(off / nt);
+  s.t0 = (int)(off % nt);
+  const long long bh_begin = bt.start[lo] + (long long)s.h * nt;
+  const long long bh_end = bh_begin + nt;
+  s.g_end = bh_end < g_limit ? bh_end : g_limit;
+  s.t1 = s.t0 + (int)(s.g_end - g);
+  s.c_first = P.cta_of(bh_begin);
+  s.c_last = P.cta_of(bh_end - 1);
+  return s;
+}
+
+// ------------------------------------------------------------------ merging
+// A partial softmax result over some keys, in the log2 domain: scores were
+// pre-multiplied by scale*log2(e); m = max, l = sum 2^(s - m), o = sum 2^(s - m) v.
+// Slot layout: nq rows of [m, l, o_0 .. o_{D-1}].
+__device__ __forceinline__ float* partial_slot(float* partials, int slot, int nq, int D) {
+  return partials + (size_t)slot * nq * (D + 2);
+}
+
+}  // namespace glide

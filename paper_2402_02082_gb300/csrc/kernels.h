@@ -1,0 +1,51 @@
+// Host-side launch interface between the C ABI (abi.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace glide {
+
+constexpr int kMaxBatch = 1024;   // sequences per call (per-CTA tile table lives in shared memory)
+constexpr int kMaxTree = 64;      // tree nodes (one 64-bit ancestor mask per node)
+constexpr int kMaxCtas = 1024;    // CTAs per attention launch (bounds the partial slots)
+
+struct AttnArgs {
+  const void* q;
+  const void* K;
+  const void* V;
+  const int32_t* kv_len;
+  const int32_t* parent;  // tree only
+  float* out;
+  void* ws;
+  int B, H, D, S_cap;
+  int nq;                 // queries per (b, h): 1 for cross-attention, n for the tree
+  int max_kv_len;
+  int dtype;              // 0 bf16, 1 f32
+  float scale;            // already resolved (never 0)
+  unsigned flags;
+  int max_ctas;           // 0 = automatic
+};
+
+struct AcceptArgs {
+  const int32_t* draft;
+  const int32_t* parent;
+  const float* logits;
+  int B, n, V;
+  int32_t* path;
+  int32_t* len;
+  int32_t* bonus;
+  void* ws;
+};
+
+int sm_count();  // multiprocessors of the current device (cached per device)
+
+cudaError_t launch_cross_attn(const AttnArgs& a, cudaStream_t st);
+cudaError_t launch_tree_attn_fma(const AttnArgs& a, cudaStream_t st);
+// Returns cudaErrorNotSupported when the tensor-core kernel does not apply to `a`.
+cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st);
+cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st);
+
+size_t accept_workspace_bytes(int B, int n);
+
+}  // namespace glide

@@ -1,0 +1,119 @@
+"""Host side of the C ABI (no GPU): the library builds and loads, exports every
+entry point include/glide.h declares, and rejects bad arguments before any
+CUDA call.  Only invalid arguments are passed here, so nothing is launched."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2402_02082_gb300 import binding as gb
+from paper_2402_02082_gb300 import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "glide.h")
+FAKE = 0x10000  # 16-byte aligned, never dereferenced: every call below fails validation first
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return gb.lib()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*[A-Za-z_][\w\s\*]*?\b([a-z_][a-z0-9_]*)\s*\(", src, flags=re.M)))
+
+
+def test_exports_every_declared_symbol(L):
+    names = declared_functions()
+    assert len(names) >= 9, names
+    for name in names:
+        assert hasattr(L, name), f"libglide.so does not export {name}"
+
+
+def test_abi_version(L):
+    assert gb.glide_abi_version() == 1
+
+
+def test_status_strings(L):
+    for s in range(5):
+        assert gb.glide_status_str(s) and gb.glide_status_str(s) != "unknown status"
+    assert gb.glide_status_str(99) == "unknown status"
+
+
+def desc(**kw):
+    d = dict(B=2, H=4, D=128, S_cap=300, dtype=gb.GLIDE_BF16, scale=0.0, flags=0, max_ctas=0)
+    d.update(kw)
+    return gb.make_desc(**d)
+
+
+def test_workspace_sizes(L):
+    d = desc()
+    w1 = gb.glide_attn_workspace_bytes(d, 1)
+    w64 = gb.glide_attn_workspace_bytes(d, 64)
+    assert 0 < w1 < w64
+    assert gb.glide_attn_workspace_bytes(d, 0) == 0
+    assert gb.glide_attn_workspace_bytes(d, 65) == 0
+    for bad in (dict(D=96), dict(B=0), dict(B=1025), dict(H=0), dict(S_cap=0), dict(dtype=7),
+                dict(scale=-1.0), dict(scale=float("nan")), dict(scale=float("inf")), dict(max_ctas=-1)):
+        assert gb.glide_attn_workspace_bytes(desc(**bad), 1) == 0, bad
+    assert gb.glide_accept_workspace_bytes(4, 64) > 0
+    assert gb.glide_accept_workspace_bytes(0, 4) == 0
+    assert gb.glide_accept_workspace_bytes(4, 65) == 0
+
+
+def cross(L, d, q=FAKE, K=FAKE, V=FAKE, kv=FAKE, max_kv=100, out=FAKE, ws=FAKE, wsb=1 << 40):
+    return L.glide_cross_attn(ctypes.byref(d), q, K, V, kv, max_kv, out, ws, wsb, None)
+
+
+def tree(L, d, n=5, q=FAKE, par=FAKE, K=FAKE, V=FAKE, kv=FAKE, max_kv=100, out=FAKE, ws=FAKE, wsb=1 << 40):
+    return L.tree_verify_attn(ctypes.byref(d), q, n, par, K, V, kv, max_kv, out, ws, wsb, None)
+
+
+def test_cross_rejects(L):
+    d = desc()
+    bad = [dict(q=None), dict(K=None), dict(V=None), dict(kv=None), dict(out=None), dict(ws=None),
+           dict(max_kv=0), dict(max_kv=301), dict(wsb=16), dict(K=FAKE + 8), dict(out=FAKE + 4),
+           dict(kv=FAKE + 2)]
+    for b in bad:
+        assert cross(L, d, **b) == gb.GLIDE_ERR_INVALID, b
+    assert cross(L, desc(D=80)) == gb.GLIDE_ERR_INVALID
+    assert L.glide_cross_attn(None, FAKE, FAKE, FAKE, FAKE, 10, FAKE, FAKE, 1 << 40, None) == gb.GLIDE_ERR_INVALID
+
+
+def test_tree_rejects(L):
+    d = desc()
+    bad = [dict(n=0), dict(n=65), dict(par=None), dict(max_kv=296), dict(max_kv=-1), dict(wsb=100),
+           dict(q=FAKE + 8), dict(par=FAKE + 1)]
+    for b in bad:
+        assert tree(L, d, **b) == gb.GLIDE_ERR_INVALID, b
+
+
+def test_accept_rejects(L):
+    def acc(draft=FAKE, par=FAKE, lg=FAKE, B=2, n=4, V=100, path=FAKE, ln=FAKE, bonus=FAKE, ws=FAKE, wsb=1 << 30):
+        return L.tree_accept(draft, par, lg, B, n, V, path, ln, bonus, ws, wsb, None)
+    for b in [dict(B=0), dict(n=0), dict(n=65), dict(V=0), dict(draft=None), dict(lg=None), dict(path=None),
+              dict(ln=None), dict(bonus=None), dict(ws=None), dict(wsb=8), dict(lg=FAKE + 4),
+              dict(path=FAKE + 2)]:
+        assert acc(**b) == gb.GLIDE_ERR_INVALID, b
+
+
+def test_validate_tree(L):
+    assert gb.glide_validate_tree(np.array([-1, 0, 1, 1, 0])) == gb.GLIDE_OK
+    assert gb.glide_validate_tree(np.array([[-1, 0, 0], [-1, 0, 1]])) == gb.GLIDE_OK
+    assert gb.glide_validate_tree(np.array([-1, 0, 2])) == gb.GLIDE_ERR_INVALID      # parent not earlier
+    assert gb.glide_validate_tree(np.array([-1, 0, -2])) == gb.GLIDE_ERR_INVALID     # below -1
+    assert gb.glide_validate_tree(np.array([0, 0, 1])) == gb.GLIDE_ERR_INVALID       # node 0 not a root
+    assert gb.glide_validate_tree(np.array([-1, 0, -1])) == gb.GLIDE_ERR_INVALID     # second root
+    assert gb.glide_validate_tree(np.array([-1, 0, -1]), require_root0=False) == gb.GLIDE_OK  # forest
+
+
+def test_binding_refuses_missing_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(gb, "_LIB", None)
+    monkeypatch.setattr(gb, "library_path", lambda: str(tmp_path / "absent.so"))
+    with pytest.raises(RuntimeError, match="not found"):
+        gb.lib()
