@@ -154,6 +154,30 @@ glide_status tree_accept(const int32_t* draft_tokens, const int32_t* parent_idx,
                          void* workspace, size_t workspace_bytes, glide_stream_t stream);
 
 /*
+ * glide_cross_attn for callers that cannot allocate device memory when they
+ * call (the paper has no counterpart; this is a deployment entry point).
+ * Examples: an engine plugin whose enqueue path must not allocate because the
+ * host engine owns and budgets all device memory, or a serving loop that has
+ * given nearly all of HBM to its KV cache and bans allocator calls on its
+ * per-token path.  Same arguments and result as glide_cross_attn, minus the
+ * workspace: the scratch lives in one fixed 4 MiB array inside the library,
+ * held on every GPU that loads the library until the process exits.
+ * - Shapes whose workspace (glide_attn_workspace_bytes(desc, 1)) exceeds
+ *   4 MiB are rejected with GLIDE_ERR_UNSUPPORTED (B*H up to 6987 for D = 128,
+ *   14640 for D = 64).
+ * - The first call on each device looks up the array's device address; make
+ *   that first call before any stream capture.
+ * - Every call first clears the words that must start at zero, then reuses the
+ *   array, so calls that overlap on the GPU (other streams, other host threads
+ *   without ordering) race on it: serialize them.
+ * - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ */
+glide_status glide_cross_attn_noalloc(const glide_attn_desc* desc, const void* q_draft,
+                                      const void* K_cache, const void* V_cache,
+                                      const int32_t* kv_len, int32_t max_kv_len, float* out,
+                                      glide_stream_t stream);
+
+/*
  * Host-side check of a parent array (HOST memory, [B,n]): every entry is -1 or
  * in [0, i).  With require_root0 != 0 (the tree_accept convention) node 0 must
  * be the only root.  Returns GLIDE_OK or GLIDE_ERR_INVALID.

@@ -52,6 +52,7 @@ _SIG = {
                                         ctypes.c_int32, _P, _P, ctypes.c_size_t, _P]),
     "tree_accept": (ctypes.c_int, [_P, _P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _P, _P, _P, _P,
                                    ctypes.c_size_t, _P]),
+    "glide_cross_attn_noalloc": (ctypes.c_int, [ctypes.POINTER(AttnDesc), _P, _P, _P, _P, ctypes.c_int32, _P, _P]),
     "glide_validate_tree": (ctypes.c_int, [_P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
     "glide_read_device_status": (ctypes.c_int, [_P, _P]),
 }
@@ -143,6 +144,24 @@ def glide_cross_attn(q_draft: torch.Tensor, K_cache: torch.Tensor, V_cache: torc
                                 kv_len.data_ptr(), int(max_kv_len), out.data_ptr(), workspace.data_ptr(),
                                 workspace.numel() * workspace.element_size(), _stream(stream))
     _check(st, "glide_cross_attn")
+    return out
+
+
+def glide_cross_attn_noalloc(q_draft: torch.Tensor, K_cache: torch.Tensor, V_cache: torch.Tensor,
+                             kv_len: torch.Tensor, max_kv_len: int, out: torch.Tensor, scale: float = 0.0,
+                             flags: int = 0, max_ctas: int = 0, stream=None) -> torch.Tensor:
+    """glide_cross_attn without a workspace, for callers that cannot allocate
+    device memory at call time; the library's fixed scratch array is used
+    (see include/glide.h for its size limit and the no-overlap rule)."""
+    desc = _cache_desc(q_draft, K_cache, V_cache, scale, flags, max_ctas)
+    if tuple(q_draft.shape) != (desc.B, 1, desc.H, desc.D) or tuple(out.shape) != (desc.B, 1, desc.H, desc.D):
+        raise ValueError("q_draft/out must be [B, 1, H, D]")
+    if out.dtype != torch.float32 or kv_len.dtype != torch.int32:
+        raise TypeError("out must be fp32 and kv_len int32")
+    st = lib().glide_cross_attn_noalloc(ctypes.byref(desc), q_draft.data_ptr(), K_cache.data_ptr(),
+                                        V_cache.data_ptr(), kv_len.data_ptr(), int(max_kv_len), out.data_ptr(),
+                                        _stream(stream))
+    _check(st, "glide_cross_attn_noalloc")
     return out
 
 
