@@ -14,6 +14,7 @@ time of the step.  --impl reference times the fp64 CPU oracle instead.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import multiprocessing as mp
@@ -182,10 +183,17 @@ def pick_pairs(w, k, seed):
 
 
 # --------------------------------------------------------------- reference
+def selected_workload(args) -> synth.Workload:
+    w = synth.workload(args.workload)
+    if args.batch and 0 < args.batch < w.B:
+        w = dataclasses.replace(w, name=f"{w.name}[:{args.batch}]", B=args.batch, kv_len=w.kv_len[:args.batch])
+    return w
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return 0
-    w = synth.workload(args.workload)
+    w = selected_workload(args)
     case = synth.make_case(w, garbage="zero")
     cores = os.cpu_count() or 1
     pool = make_pool(cores)
@@ -234,7 +242,7 @@ def run_glide(args, rank, world, local_rank):
     build.build()
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    w = synth.workload(args.workload)
+    w = selected_workload(args)
 
     cpu = None
     if world == 1 and rank == 0 and not args.no_cpu_baseline:
@@ -437,6 +445,8 @@ def main():
     ap.add_argument("--cpu-pairs", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--force-fma", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="keep only the first N sequences of the workload (smaller profiling captures)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -1,9 +1,481 @@
-// Tree verification attention on the tcgen05 tensor cores.
-// Not yet available: every call falls back to the CUDA-core kernel.
+// Tree verification attention on the tcgen05 tensor cores (Section 3.2:
+// the CaPE verification mask, here as the general ancestor-or-self mask of a
+// linearized token tree).  bf16 Q/K/V, fp32 accumulation, D in {64, 128},
+// n <= 64 tree queries per (sequence, head).
+//
+// At n = 26..64 queries the verification does n flops per KV byte, beyond
+// what CUDA-core FMA can sustain at HBM speed, so both products run on the
+// tensor cores while the KV stream stays the bound:
+//   S = Q K^T   : M = 128 (queries, zero-padded), N = 64 keys, K = D
+//   O += P V    : M = 128, N = D, K = 64 keys
+// Operands sit in shared memory in the 128-byte-swizzled K-major layout
+// (Q, K, P) or M/N-major layout (V), accumulators in tensor memory (TMEM):
+// two S buffers of 64 columns and O of D columns, 256 columns in all.
+//
+// Roles (192 threads, persistent grid of one CTA per SM, split-KV partition
+// shared with the other attention kernels):
+//   warps 0-3  softmax: thread r owns query row r (= TMEM lane r); reads S,
+//              masks, keeps the running max and sum, writes P (bf16) to
+//              shared memory, rescales O in TMEM when the max grows, and
+//              finishes each segment (normalize, or write a split partial);
+//   warp 4     producer: one thread loads K and V tiles with 2-D TMA
+//              (64 keys x 64 head dims per box, 128-byte swizzle);
+//   warp 5     MMA: allocates TMEM; one thread issues S(j+1) before PV(j) so
+//              the softmax of one tile overlaps the P.V product of the last.
+//
+// Online softmax in the log2 domain with a lazy reference max: the max used
+// for the exponent only moves when a tile's max exceeds it by more than 8
+// (factor 256), so O is rescaled in TMEM rarely; the final division by the
+// sum taken with the same reference makes the result exact up to rounding.
+// V rows past the end of a slab are zeroed in shared memory before P.V (the
+// cache beyond kv_len + n may hold anything, even NaN).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <math_constants.h>
+
+#include <mutex>
+
+#include "attn_common.cuh"
 #include "kernels.h"
+#include "tc_ptx.cuh"
 
 namespace glide {
+namespace {
 
-cudaError_t launch_tree_attn_tc(const AttnArgs&, cudaStream_t) { return cudaErrorNotSupported; }
+constexpr int kTK = 64;          // keys per tile
+constexpr int kM = 128;          // MMA rows
+constexpr int kStages = 4;       // K/V stages
+constexpr int kThreads = 192;
+constexpr int kProdWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kSoft = 128;       // softmax threads
+constexpr uint32_t kTmemCols = 256;
+constexpr float kRescaleLog2 = 8.0f;
+
+// barrier slots
+constexpr int B_KFULL = 0, B_VFULL = 4, B_KEMPTY = 8, B_VEMPTY = 12, B_SFULL = 16, B_SFREE = 18, B_PFULL = 20,
+              B_PFREE = 22, B_ODONE = 24, B_OFREE = 26, B_QFULL = 27, B_MDONE = 28, kNumBars = 29;
+
+template <int D>
+struct TcCfg {
+  static constexpr int kHalves = D / 64;              // 128-byte swizzle atoms across the head dim
+  static constexpr uint32_t kQHalf = kM * 128;        // 128 rows x 128 B
+  static constexpr uint32_t kQBytes = kHalves * kQHalf;
+  static constexpr uint32_t kPBytes = kM * kTK * 2;   // 128 rows x 64 keys bf16
+  static constexpr uint32_t kKVHalf = kTK * 128;      // 64 keys x 128 B
+  static constexpr uint32_t kKVTile = kHalves * kKVHalf;
+  static constexpr uint32_t off_Q = 0;
+  static constexpr uint32_t off_P = off_Q + kQBytes;
+  static constexpr uint32_t off_K = off_P + 2 * kPBytes;
+  static constexpr uint32_t off_V = off_K + kStages * kKVTile;
+  static constexpr uint32_t off_bar = off_V + kStages * kKVTile;
+  static constexpr uint32_t off_misc = off_bar + 256;
+  static constexpr uint32_t off_tab = off_misc + 32;
+  static constexpr uint32_t kTmemO = 2 * kTK;          // S buffers at columns 0 and 64, O after them
+  static_assert(kNumBars * 8 <= 256, "barrier area");
+  static_assert(kTmemO + D <= kTmemCols, "TMEM columns");
+  static size_t smem_bytes(int B) { return 1024 + off_tab + (size_t)(B + 1) * 8 + (size_t)3 * B * 4; }
+};
+
+struct TcParams {
+  const __nv_bfloat16* q;
+  const int* kv_len;
+  const int* parent;
+  float* out;
+  unsigned* status;
+  unsigned* counters;
+  float* partials;
+  int B, H, S_cap, max_kv_len, n;
+  float scale_log2;
+};
+
+// Lane 0 waits, the warp follows: every lane sees the same outcome, so the
+// warp-collective tcgen05 instructions that follow stay convergent.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, unsigned* status) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, status) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                        const TcParams p) {
+  using C = TcCfg<D>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc + 4);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(base + C::off_misc + 8);
+  BatchTiles bt;
+  bt.start = reinterpret_cast<long long*>(base + C::off_tab);
+  bt.len = reinterpret_cast<int*>(bt.start + p.B + 1);
+  bt.ntiles = bt.len + p.B;
+  bt.plen = bt.ntiles + p.B;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = p.n;
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < kNumBars; ++b) {
+      uint32_t cnt = 1;
+      if (b == B_SFREE || b == B_SFREE + 1 || b == B_PFULL || b == B_PFULL + 1 || b == B_OFREE || b == B_QFULL)
+        cnt = 4;  // one arrival per softmax warp
+      mbar_init(&bars[b], cnt);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kMmaWarp) {
+    tc::tmem_alloc(tmem_slot, kTmemCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  build_batch_tiles(bt, p.kv_len, p.B, p.H, p.max_kv_len, n, kTK);  // __syncthreads inside
+  tc::fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  Partition P;
+  P.init(bt.start[p.B], gridDim.x);
+  const long long g_begin = P.begin(blockIdx.x), g_end = P.end(blockIdx.x);
+
+  if (warp == kProdWarp) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmK);
+      tc::prefetch_tmap(&tmV);
+      const uint64_t pol = policy_evict_first();
+      int i = 0, nk = 0, nv = 0;
+      bool ok = true;
+      for (long long g = g_begin; g < g_end && ok;) {
+        const Segment s = locate(bt, P, p.B, g, g_end);
+        const int slab_row = (s.b * p.H + s.h) * p.S_cap;
+        for (int t = s.t0; t < s.t1; ++t, ++i) {
+          const int st = i % kStages;
+          const uint32_t ph = (i / kStages) & 1;
+          if (!mbar_wait(&bars[B_KEMPTY + st], ph ^ 1, abort_flag, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&bars[B_KFULL + st], C::kKVTile);
+          for (int hd = 0; hd < C::kHalves; ++hd)
+            tc::tma_load_2d(base + C::off_K + st * C::kKVTile + hd * C::kKVHalf, &tmK, hd * 64, slab_row + t * kTK,
+                            &bars[B_KFULL + st], pol);
+          ++nk;
+          if (!mbar_wait(&bars[B_VEMPTY + st], ph ^ 1, abort_flag, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&bars[B_VFULL + st], C::kKVTile);
+          for (int hd = 0; hd < C::kHalves; ++hd)
+            tc::tma_load_2d(base + C::off_V + st * C::kKVTile + hd * C::kKVHalf, &tmV, hd * 64, slab_row + t * kTK,
+                            &bars[B_VFULL + st], pol);
+          ++nv;
+        }
+        g = s.g_end;
+      }
+      if (!ok) {  // let issued loads land before the CTA exits
+        for (int j = (nk > kStages ? nk - kStages : 0); j < nk; ++j)
+          mbar_drain(&bars[B_KFULL + j % kStages], (j / kStages) & 1);
+        for (int j = (nv > kStages ? nv - kStages : 0); j < nv; ++j)
+          mbar_drain(&bars[B_VFULL + j % kStages], (j / kStages) & 1);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ----------------------------------------------------------------- MMA
+    if (lane == 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(kM, kTK, false, false);
+      constexpr uint32_t idO = tc::idesc_bf16_f32(kM, D, false, true);
+      const uint32_t sQ = smem_u32(base + C::off_Q), sP = smem_u32(base + C::off_P);
+      const uint32_t sK = smem_u32(base + C::off_K), sV = smem_u32(base + C::off_V);
+      int i = 0, seg = 0;
+      bool ok = true;
+      auto issue_pv = [&](int jj, bool first_in_seg) -> bool {
+        if (!mbar_wait(&bars[B_PFULL + (jj & 1)], (jj >> 1) & 1, abort_flag, p.status)) return false;
+        if (!mbar_wait(&bars[B_VFULL + jj % kStages], (jj / kStages) & 1, abort_flag, p.status)) return false;
+        if (first_in_seg && seg > 0 && !mbar_wait(&bars[B_OFREE], (seg - 1) & 1, abort_flag, p.status)) return false;
+        tc::fence_after_sync();
+        const uint32_t vb = sV + (jj % kStages) * C::kKVTile;
+        const uint32_t pb = sP + (jj & 1) * C::kPBytes;
+#pragma unroll
+        for (int ks = 0; ks < kTK / 16; ++ks) {
+          const uint64_t a = tc::sw128_desc(pb + ks * 32, 16, 1024);
+          const uint64_t bdesc = tc::sw128_desc(vb + ks * 16 * 128, C::kKVHalf, 1024);
+          tc::mma_bf16(tmem + C::kTmemO, a, bdesc, idO, (first_in_seg && ks == 0) ? 0u : 1u);
+        }
+        tc::mma_commit(&bars[B_PFREE + (jj & 1)]);
+        tc::mma_commit(&bars[B_VEMPTY + jj % kStages]);
+        tc::mma_commit(&bars[B_ODONE + (jj & 1)]);
+        return true;
+      };
+      for (long long g = g_begin; g < g_end && ok;) {
+        const Segment s = locate(bt, P, p.B, g, g_end);
+        if (!mbar_wait(&bars[B_QFULL], seg & 1, abort_flag, p.status)) { ok = false; break; }
+        for (int t = s.t0; t < s.t1; ++t, ++i) {
+          const int j = i;
+          if (!mbar_wait(&bars[B_KFULL + j % kStages], (j / kStages) & 1, abort_flag, p.status) ||
+              !mbar_wait(&bars[B_SFREE + (j & 1)], ((j >> 1) & 1) ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t kb = sK + (j % kStages) * C::kKVTile;
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const uint64_t a = tc::sw128_desc(sQ + (ks / 4) * C::kQHalf + (ks % 4) * 32, 16, 1024);
+            const uint64_t bdesc = tc::sw128_desc(kb + (ks / 4) * C::kKVHalf + (ks % 4) * 32, 16, 1024);
+            tc::mma_bf16(tmem + (j & 1) * kTK, a, bdesc, idS, ks > 0 ? 1u : 0u);
+          }
+          tc::mma_commit(&bars[B_SFULL + (j & 1)]);
+          tc::mma_commit(&bars[B_KEMPTY + j % kStages]);
+          if (t > s.t0 && !issue_pv(j - 1, t - 1 == s.t0)) { ok = false; break; }
+        }
+        if (ok && !issue_pv(i - 1, s.t1 - 1 == s.t0)) ok = false;
+        ++seg;
+        g = s.g_end;
+      }
+      tc::mma_commit(&bars[B_MDONE]);  // every MMA finished before TMEM is released
+      mbar_drain(&bars[B_MDONE], 0);
+    }
+  } else {
+    // ------------------------------------------------------------- softmax
+    const int row = threadIdx.x;  // query row = TMEM lane
+    const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
+    const float sl2 = p.scale_log2;
+    bool dead = false;
+    int i = 0;
+    for (long long g = g_begin; g < g_end;) {
+      const Segment s = locate(bt, P, p.B, g, g_end);
+      const int plen = bt.plen[s.b], len = bt.len[s.b];
+
+      // this segment's queries into the swizzled Q tile (rows >= n are zero)
+      {
+        unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
+        const uint4* src = reinterpret_cast<const uint4*>(p.q + (((size_t)s.b * n + (row < n ? row : 0)) * p.H +
+                                                                  s.h) * D);
+#pragma unroll
+        for (int hd = 0; hd < C::kHalves; ++hd)
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            uint4 v = make_uint4(0u, 0u, 0u, 0u);
+            if (row < n) v = src[hd * 8 + c];
+            *reinterpret_cast<uint4*>(qrow + hd * C::kQHalf + ((c ^ (row & 7)) << 4)) = v;
+          }
+      }
+      uint64_t anc = 0;  // ancestor-or-self set of this row's node
+      if (row < n) {
+        int j = row;
+        for (int step = 0; step < kMaxTree && j >= 0; ++step) {
+          anc |= 1ull << j;
+          const int pj = p.parent[(size_t)s.b * n + j];
+          j = (pj >= 0 && pj < j) ? pj : -1;
+        }
+      }
+      tc::fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_QFULL]);
+
+      float m_used = -CUDART_INF_F, l = 0.f;
+      for (int t = s.t0; t < s.t1; ++t, ++i) {
+        const int j = i;
+        uint32_t sr[2][32];
+        if (!dead) dead = !warp_wait(&bars[B_SFULL + (j & 1)], (j >> 1) & 1, abort_flag, p.status);
+        if (!dead) {
+          tc::fence_after_sync();
+          tc::tmem_ld32(lane_addr + (j & 1) * kTK, sr[0]);
+          tc::tmem_ld32(lane_addr + (j & 1) * kTK + 32, sr[1]);
+          tc::tmem_wait_ld();
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_SFREE + (j & 1)]);
+
+        // scores in the log2 domain, masked
+        const int key0 = t * kTK;
+        float sc[kTK];
+        float tmax = -CUDART_INF_F;
+        const bool all_prefix = key0 + kTK <= plen;
+#pragma unroll
+        for (int k = 0; k < kTK; ++k) {
+          const int key = key0 + k;
+          const bool vis = all_prefix || (key < len && (key < plen || ((anc >> ((key - plen) & 63)) & 1ull)));
+          sc[k] = vis ? __uint_as_float(sr[k >> 5][k & 31]) * sl2 : -CUDART_INF_F;
+          tmax = fmaxf(tmax, sc[k]);
+        }
+        const bool need = tmax > m_used + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float m_new = need ? tmax : m_used;
+          const float f = need ? fast_exp2(m_used - m_new) : 1.f;
+          l *= f;
+          if (t > s.t0 && !dead) {  // O holds the P.V of earlier tiles of this segment
+            dead = !warp_wait(&bars[B_ODONE + ((j - 1) & 1)], ((j - 1) >> 1) & 1, abort_flag, p.status);
+            if (!dead) {
+              tc::fence_after_sync();
+#pragma unroll 1
+              for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tc::tmem_ld32(lane_addr + C::kTmemO + c * 32, o);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
+                tc::tmem_st32(lane_addr + C::kTmemO + c * 32, o);
+              }
+              tc::tmem_wait_st();
+            }
+          }
+          m_used = m_new;
+        }
+        const float m_eff = m_used == -CUDART_INF_F ? 0.f : m_used;
+        uint32_t pk[kTK / 2];
+        float lsum = 0.f;
+#pragma unroll
+        for (int k = 0; k < kTK / 2; ++k) {
+          const float p0 = fast_exp2(sc[2 * k] - m_eff);
+          const float p1 = fast_exp2(sc[2 * k + 1] - m_eff);
+          lsum += p0 + p1;
+          pk[k] = pack_bf16x2(p0, p1);
+        }
+        l += lsum;
+
+        if (!dead) dead = !warp_wait(&bars[B_PFREE + (j & 1)], ((j >> 1) & 1) ^ 1, abort_flag, p.status);
+        {
+          unsigned char* prow = base + C::off_P + (j & 1) * C::kPBytes + (row >> 3) * 1024 + (row & 7) * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) =
+                make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        }
+        const int vrows = len - key0;
+        if (vrows < kTK) {  // last tile of the slab: clear V rows past its end
+          const int st = j % kStages;
+          if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (j / kStages) & 1, abort_flag, p.status);
+          for (int idx = row; idx < (kTK - vrows) * C::kHalves; idx += kSoft) {
+            const int r = vrows + idx / C::kHalves, hd = idx % C::kHalves;
+            uint4* dst = reinterpret_cast<uint4*>(base + C::off_V + st * C::kKVTile + hd * C::kKVHalf + r * 128);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
+          }
+        }
+        tc::fence_async_smem();
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_PFULL + (j & 1)]);
+      }
+
+      // ---- segment epilogue: O / l, or a split partial
+      const int jl = i - 1;
+      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+      const bool single = s.c_first == s.c_last;
+      const int bh = s.b * p.H + s.h;
+      float* dst = single ? p.out + (((size_t)s.b * n + row) * p.H + s.h) * D
+                          : partial_slot(p.partials, blockIdx.x + bh, n, D) + (size_t)row * (D + 2);
+      if (!dead) {
+        tc::fence_after_sync();
+        const float inv = single ? 1.f / l : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tc::tmem_ld32(lane_addr + C::kTmemO + c * 32, o);
+          tc::tmem_wait_ld();
+          if (row < n) {
+            float* d = dst + (single ? 0 : 2) + c * 32;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) d[k] = __uint_as_float(o[k]) * inv;
+          }
+        }
+        if (!single && row < n) {
+          dst[0] = m_used;
+          dst[1] = l;
+        }
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_OFREE]);
+      if (!single) combine_if_last(s, p.B, p.H, n, D, p.partials, p.counters, p.out, row, kSoft, last_flag);
+      g = s.g_end;
+    }
+  }
+
+  __syncwarp();  // the producer and MMA warps reconverge after their single-lane loops
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------- host
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// [rows, D] bf16 view of a K or V cache; boxes of 64 head dims x 64 keys, 128-byte swizzle.
+bool make_kv_map(CUtensorMap* m, const void* base, long long rows, int D) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kTK};
+  const cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D>
+cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
+  using C = TcCfg<D>;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)C::smem_bytes(kMaxBatch));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  const long long rows = (long long)a.B * a.H * a.S_cap;
+  CUtensorMap mk, mv;
+  if (!make_kv_map(&mk, a.K, rows, D) || !make_kv_map(&mv, a.V, rows, D)) return cudaErrorNotSupported;
+  const long long tiles_ub = (long long)a.B * a.H * ((a.max_kv_len + a.nq + kTK - 1) / kTK);
+  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
+  if (G > kMaxCtas) G = kMaxCtas;
+  if (G > tiles_ub) G = tiles_ub;
+  if (G < 1) G = 1;
+  TcParams p;
+  p.q = static_cast<const __nv_bfloat16*>(a.q);
+  p.kv_len = a.kv_len;
+  p.parent = a.parent;
+  p.out = a.out;
+  unsigned char* ws = static_cast<unsigned char*>(a.ws);
+  p.status = reinterpret_cast<unsigned*>(ws);
+  p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
+  p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
+  p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
+  p.scale_log2 = a.scale * kLog2e;
+  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B), st>>>(mk, mv, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st) {
+  if (a.dtype != 0 || (a.D != 128 && a.D != 64)) return cudaErrorNotSupported;
+  if ((long long)a.B * a.H * a.S_cap > 0x7fffffffLL) return cudaErrorNotSupported;  // 32-bit TMA row coordinate
+  if (a.D == 128) return launch_typed<128>(a, st);
+  return launch_typed<64>(a, st);
+}
 
 }  // namespace glide
