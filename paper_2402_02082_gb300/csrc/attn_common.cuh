@@ -52,6 +52,22 @@ __device__ __forceinline__ float transpose_reduce32(float (&part)[32], int lane)
   return part[0];
 }
 
+// The same for 16 keys: four exchange rounds and one final pairwise sum leave
+// lanes 2k and 2k+1 both holding the full sum for key k (16 shuffles).
+__device__ __forceinline__ float transpose_reduce16(float (&part)[16], int lane) {
+#pragma unroll
+  for (int off = 16, cnt = 8; off >= 2; off >>= 1, cnt >>= 1) {
+    const bool upper = (lane & off) != 0;
+#pragma unroll
+    for (int j = 0; j < cnt; ++j) {
+      const float send = upper ? part[j] : part[j + cnt];
+      const float keep = upper ? part[j + cnt] : part[j];
+      part[j] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+    }
+  }
+  return part[0] + __shfl_xor_sync(0xffffffffu, part[0], 1);
+}
+
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
   for (int off = 16; off >= 1; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));

@@ -6,17 +6,18 @@
 // The step reads every cached K and V byte once and does ~1 flop per byte, so
 // it is bound by HBM bandwidth.  Design:
 // * persistent grid (one CTA per SM); the key ranges of all (b, h) are cut
-//   into 32-key tiles and dealt to CTAs in equal contiguous shares (split-KV
+//   into 16-key tiles and dealt to CTAs in equal contiguous shares (split-KV
 //   with exact balance, ragged batches included);
 // * one producer thread streams K and V tiles with 1-D bulk copies (TMA) into
 //   shared-memory stages guarded by mbarriers; tile i goes to consumer warp
 //   i % NW, and every consumer warp owns a private ring of SW stages that it
 //   drains strictly in order (a warp never waits on a stage whose earlier
 //   phase is still pending, so the mbarrier parity cannot alias);
-// * each of the NW consumer warps takes whole tiles: lanes split the head
-//   dimension, a transpose-reduction turns 32x(D/32)-element partial dot
-//   products into one score per lane, and an fp32 online softmax (log2
-//   domain) accumulates P.V;
+// * each of the NW = 8 consumer warps (two per SM sub-partition, so one
+//   warp's shuffle and shared-memory latencies hide behind the other's work)
+//   takes whole tiles: lanes split the head dimension, a transpose-reduction
+//   turns 16x(D/32)-element partial dot products into one score per lane pair,
+//   and an fp32 online softmax (log2 domain) accumulates P.V;
 // * per segment the warps merge in shared memory; a (b, h) split across CTAs
 //   is finished by the last CTA to arrive (atomic counter, no waiting).
 #include <cuda_bf16.h>
@@ -28,8 +29,8 @@
 namespace glide {
 namespace {
 
-constexpr int kTK = 32;      // keys per tile
-constexpr int kNW = 4;       // consumer warps
+constexpr int kTK = 16;      // keys per tile
+constexpr int kNW = 8;       // consumer warps
 constexpr int kThreads = (kNW + 1) * 32;
 
 template <typename T, int D>
@@ -168,9 +169,9 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
       const T* Kt = sK + (size_t)st * kTK * D + lane * E;
       const T* Vt = sV + (size_t)st * kTK * D + lane * E;
 
-      float part[32];
+      float part[kTK];
 #pragma unroll
-      for (int k = 0; k < 32; ++k) {
+      for (int k = 0; k < kTK; ++k) {
         float kf[E];
         load_row_chunk<T, E>(Kt + k * D, kf);
         float acc = 0.f;
@@ -178,18 +179,18 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
         for (int e = 0; e < E; ++e) acc = fmaf(q[e], kf[e], acc);
         part[k] = acc;
       }
-      float sc = transpose_reduce32(part, lane);
-      if (lane >= rows) sc = -CUDART_INF_F;
+      float sc = transpose_reduce16(part, lane);  // score of key lane / 2
+      if ((lane >> 1) >= rows) sc = -CUDART_INF_F;
       const float m_new = fmaxf(m, warp_max(sc));
       const float corr = fast_exp2(m - m_new);
       const float pe = fast_exp2(sc - m_new);
-      l = l * corr + pe;
+      l = l * corr + ((lane & 1) ? 0.f : pe);  // each key is held by two lanes: count it once
 #pragma unroll
       for (int e = 0; e < E; ++e) o[e] *= corr;
 #pragma unroll
-      for (int k = 0; k < 32; ++k) {
+      for (int k = 0; k < kTK; ++k) {
         if (k < rows) {
-          const float pk = __shfl_sync(0xffffffffu, pe, k);
+          const float pk = __shfl_sync(0xffffffffu, pe, 2 * k);
           float vf[E];
           load_row_chunk<T, E>(Vt + k * D, vf);
 #pragma unroll

@@ -6,21 +6,25 @@
 // At n = 26..64 queries the verification does n flops per KV byte, beyond
 // what CUDA-core FMA can sustain at HBM speed, so both products run on the
 // tensor cores while the KV stream stays the bound:
-//   S = Q K^T   : M = 128 (queries, zero-padded), N = 64 keys, K = D
-//   O += P V    : M = 128, N = D, K = 64 keys
+//   S = Q K^T   : M = 128 (query rows, zero-padded), N = 64 keys, K = D
+//   O += P V    : M = 128, N = D, K = 32 keys, once per key half
 // Operands sit in shared memory in the 128-byte-swizzled K-major layout
-// (Q, K, P) or M/N-major layout (V), accumulators in tensor memory (TMEM):
-// two S buffers of 64 columns and O of D columns, 256 columns in all.
+// (Q, K, P) or M/N-major layout (V); accumulators live in tensor memory
+// (TMEM): two S buffers of 64 columns and one O accumulator of D columns for
+// each key half.
 //
-// Roles (192 threads, persistent grid of one CTA per SM, split-KV partition
+// Roles (320 threads, persistent grid of one CTA per SM, split-KV partition
 // shared with the other attention kernels):
-//   warps 0-3  softmax: thread r owns query row r (= TMEM lane r); reads S,
-//              masks, keeps the running max and sum, writes P (bf16) to
-//              shared memory, rescales O in TMEM when the max grows, and
-//              finishes each segment (normalize, or write a split partial);
-//   warp 4     producer: one thread loads K and V tiles with 2-D TMA
-//              (64 keys x 64 head dims per box, 128-byte swizzle);
-//   warp 5     MMA: allocates TMEM; one thread issues S(j+1) before PV(j) so
+//   warps 0-7  softmax.  Warp w reads TMEM lane quarter w % 4 (32 query
+//              rows) and key half w / 4 (32 of the tile's 64 keys).  Each
+//              (row, key half) keeps its own running max and sum and its own
+//              O accumulator, so no values cross warps inside the key loop;
+//              the halves are merged once per segment.  Query i sits in row
+//              (i % 4) * 32 + i / 4, which spreads any tree over all four
+//              lane quarters (all four SM sub-partitions).
+//   warp 8     producer: lane 0 loads K tiles, lane 1 V tiles, with 2-D TMA
+//              (64 keys x 64 head dims per box, 128-byte swizzle).
+//   warp 9     MMA: allocates TMEM; one thread issues S(j+1) before PV(j) so
 //              the softmax of one tile overlaps the P.V product of the last.
 //
 // Online softmax in the log2 domain with a lazy reference max: the max used
@@ -44,13 +48,13 @@ namespace glide {
 namespace {
 
 constexpr int kTK = 64;          // keys per tile
+constexpr int kHK = 32;          // keys per key half
 constexpr int kM = 128;          // MMA rows
 constexpr int kStages = 4;       // K/V stages
-constexpr int kThreads = 192;
-constexpr int kProdWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kSoft = 128;       // softmax threads
-constexpr uint32_t kTmemCols = 256;
+constexpr int kSoftWarps = 8;
+constexpr int kProdWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kThreads = 320;
 constexpr float kRescaleLog2 = 8.0f;
 
 // barrier slots
@@ -70,11 +74,12 @@ struct TcCfg {
   static constexpr uint32_t off_K = off_P + 2 * kPBytes;
   static constexpr uint32_t off_V = off_K + kStages * kKVTile;
   static constexpr uint32_t off_bar = off_V + kStages * kKVTile;
-  static constexpr uint32_t off_misc = off_bar + 256;
+  static constexpr uint32_t off_ml = off_bar + 256;                // [128] (max, sum) of key half 1
+  static constexpr uint32_t off_misc = off_ml + kM * 8;
   static constexpr uint32_t off_tab = off_misc + 32;
-  static constexpr uint32_t kTmemO = 2 * kTK;          // S buffers at columns 0 and 64, O after them
+  static constexpr uint32_t kTmemO = 2 * kTK;                      // S buffers at columns 0 and 64
+  static constexpr uint32_t kTmemCols = kTmemO + 2 * D <= 256 ? 256 : 512;
   static_assert(kNumBars * 8 <= 256, "barrier area");
-  static_assert(kTmemO + D <= kTmemCols, "TMEM columns");
   static size_t smem_bytes(int B) { return 1024 + off_tab + (size_t)(B + 1) * 8 + (size_t)3 * B * 4; }
 };
 
@@ -106,6 +111,9 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+// Named barrier among the 256 softmax threads (id 2; id 1 belongs to the split merge).
+__device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -114,6 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ unsigned char smem_raw[];
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar);
+  float2* ml = reinterpret_cast<float2*>(base + C::off_ml);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc + 4);
   volatile int* last_flag = reinterpret_cast<volatile int*>(base + C::off_misc + 8);
@@ -128,15 +137,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int b = 0; b < kNumBars; ++b) {
       uint32_t cnt = 1;
-      if (b == B_SFREE || b == B_SFREE + 1 || b == B_PFULL || b == B_PFULL + 1 || b == B_OFREE || b == B_QFULL)
-        cnt = 4;  // one arrival per softmax warp
+      if (b == B_SFREE || b == B_SFREE + 1 || b == B_PFULL || b == B_PFULL + 1) cnt = kSoftWarps;
+      if (b == B_OFREE || b == B_QFULL) cnt = 4;  // the key-half-0 warps
       mbar_init(&bars[b], cnt);
     }
     *abort_flag = 0;
     fence_barrier_init();
   }
   if (warp == kMmaWarp) {
-    tc::tmem_alloc(tmem_slot, kTmemCols);
+    tc::tmem_alloc(tmem_slot, C::kTmemCols);
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
@@ -150,38 +159,30 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kProdWarp) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmK);
-      tc::prefetch_tmap(&tmV);
+    if (lane < 2) {  // lane 0: K tiles, lane 1: V tiles
+      const CUtensorMap* map = lane == 0 ? &tmK : &tmV;
+      uint64_t* full = &bars[lane == 0 ? B_KFULL : B_VFULL];
+      uint64_t* empty = &bars[lane == 0 ? B_KEMPTY : B_VEMPTY];
+      const uint32_t dst0 = lane == 0 ? C::off_K : C::off_V;
+      tc::prefetch_tmap(map);
       const uint64_t pol = policy_evict_first();
-      int i = 0, nk = 0, nv = 0;
+      int i = 0;
       bool ok = true;
       for (long long g = g_begin; g < g_end && ok;) {
         const Segment s = locate(bt, P, p.B, g, g_end);
         const int slab_row = (s.b * p.H + s.h) * p.S_cap;
         for (int t = s.t0; t < s.t1; ++t, ++i) {
           const int st = i % kStages;
-          const uint32_t ph = (i / kStages) & 1;
-          if (!mbar_wait(&bars[B_KEMPTY + st], ph ^ 1, abort_flag, p.status)) { ok = false; break; }
-          mbar_arrive_expect_tx(&bars[B_KFULL + st], C::kKVTile);
+          if (!mbar_wait(&empty[st], ((i / kStages) & 1) ^ 1, abort_flag, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[st], C::kKVTile);
           for (int hd = 0; hd < C::kHalves; ++hd)
-            tc::tma_load_2d(base + C::off_K + st * C::kKVTile + hd * C::kKVHalf, &tmK, hd * 64, slab_row + t * kTK,
-                            &bars[B_KFULL + st], pol);
-          ++nk;
-          if (!mbar_wait(&bars[B_VEMPTY + st], ph ^ 1, abort_flag, p.status)) { ok = false; break; }
-          mbar_arrive_expect_tx(&bars[B_VFULL + st], C::kKVTile);
-          for (int hd = 0; hd < C::kHalves; ++hd)
-            tc::tma_load_2d(base + C::off_V + st * C::kKVTile + hd * C::kKVHalf, &tmV, hd * 64, slab_row + t * kTK,
-                            &bars[B_VFULL + st], pol);
-          ++nv;
+            tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, slab_row + t * kTK,
+                            &full[st], pol);
         }
         g = s.g_end;
       }
       if (!ok) {  // let issued loads land before the CTA exits
-        for (int j = (nk > kStages ? nk - kStages : 0); j < nk; ++j)
-          mbar_drain(&bars[B_KFULL + j % kStages], (j / kStages) & 1);
-        for (int j = (nv > kStages ? nv - kStages : 0); j < nv; ++j)
-          mbar_drain(&bars[B_VFULL + j % kStages], (j / kStages) & 1);
+        for (int j = (i > kStages ? i - kStages : 0); j < i; ++j) mbar_drain(&full[j % kStages], (j / kStages) & 1);
       }
     }
   } else if (warp == kMmaWarp) {
@@ -193,6 +194,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t sK = smem_u32(base + C::off_K), sV = smem_u32(base + C::off_V);
       int i = 0, seg = 0;
       bool ok = true;
+      // O_h += P[:, 32h .. 32h+31] V[32h .. 32h+31, :] for key halves h = 0, 1
       auto issue_pv = [&](int jj, bool first_in_seg) -> bool {
         if (!mbar_wait(&bars[B_PFULL + (jj & 1)], (jj >> 1) & 1, abort_flag, p.status)) return false;
         if (!mbar_wait(&bars[B_VFULL + jj % kStages], (jj / kStages) & 1, abort_flag, p.status)) return false;
@@ -202,9 +204,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t pb = sP + (jj & 1) * C::kPBytes;
 #pragma unroll
         for (int ks = 0; ks < kTK / 16; ++ks) {
+          const int h = ks >> 1;
           const uint64_t a = tc::sw128_desc(pb + ks * 32, 16, 1024);
           const uint64_t bdesc = tc::sw128_desc(vb + ks * 16 * 128, C::kKVHalf, 1024);
-          tc::mma_bf16(tmem + C::kTmemO, a, bdesc, idO, (first_in_seg && ks == 0) ? 0u : 1u);
+          tc::mma_bf16(tmem + C::kTmemO + h * D, a, bdesc, idO, (first_in_seg && (ks & 1) == 0) ? 0u : 1u);
         }
         tc::mma_commit(&bars[B_PFREE + (jj & 1)]);
         tc::mma_commit(&bars[B_VEMPTY + jj % kStages]);
@@ -242,8 +245,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------- softmax
-    const int row = threadIdx.x;  // query row = TMEM lane
-    const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
+    const int quarter = warp & 3, half = warp >> 2;
+    const int row = quarter * 32 + lane;       // TMEM lane = MMA row
+    const int qi = lane * 4 + quarter;         // the tree query in this row
+    const bool valid = qi < n;
+    const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+    const uint32_t o_col = C::kTmemO + half * D;
+    const int sid = threadIdx.x;               // 0..255 among the softmax threads
     const float sl2 = p.scale_log2;
     bool dead = false;
     int i = 0;
@@ -251,60 +259,66 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Segment s = locate(bt, P, p.B, g, g_end);
       const int plen = bt.plen[s.b], len = bt.len[s.b];
 
-      // this segment's queries into the swizzled Q tile (rows >= n are zero)
-      {
+      if (half == 0) {
+        // this segment's queries into the swizzled Q tile (padding rows are zero)
         unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
-        const uint4* src = reinterpret_cast<const uint4*>(p.q + (((size_t)s.b * n + (row < n ? row : 0)) * p.H +
-                                                                  s.h) * D);
+        const uint4* src =
+            reinterpret_cast<const uint4*>(p.q + (((size_t)s.b * n + (valid ? qi : 0)) * p.H + s.h) * D);
 #pragma unroll
         for (int hd = 0; hd < C::kHalves; ++hd)
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
             uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (row < n) v = src[hd * 8 + c];
+            if (valid) v = src[hd * 8 + c];
             *reinterpret_cast<uint4*>(qrow + hd * C::kQHalf + ((c ^ (row & 7)) << 4)) = v;
           }
+        tc::fence_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_QFULL]);
       }
-      uint64_t anc = 0;  // ancestor-or-self set of this row's node
-      if (row < n) {
-        int j = row;
+      uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
+      if (valid) {
+        int j = qi;
         for (int step = 0; step < kMaxTree && j >= 0; ++step) {
           anc |= 1ull << j;
           const int pj = p.parent[(size_t)s.b * n + j];
           j = (pj >= 0 && pj < j) ? pj : -1;
         }
       }
-      tc::fence_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars[B_QFULL]);
 
       float m_used = -CUDART_INF_F, l = 0.f;
       for (int t = s.t0; t < s.t1; ++t, ++i) {
         const int j = i;
-        uint32_t sr[2][32];
+        uint32_t sr[32];
         if (!dead) dead = !warp_wait(&bars[B_SFULL + (j & 1)], (j >> 1) & 1, abort_flag, p.status);
         if (!dead) {
           tc::fence_after_sync();
-          tc::tmem_ld32(lane_addr + (j & 1) * kTK, sr[0]);
-          tc::tmem_ld32(lane_addr + (j & 1) * kTK + 32, sr[1]);
+          tc::tmem_ld32(lane_addr + (j & 1) * kTK + half * kHK, sr);
           tc::tmem_wait_ld();
         }
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars[B_SFREE + (j & 1)]);
 
-        // scores in the log2 domain, masked
-        const int key0 = t * kTK;
-        float sc[kTK];
-        float tmax = -CUDART_INF_F;
-        const bool all_prefix = key0 + kTK <= plen;
+        // scores of this key half in the log2 domain, masked
+        const int key0 = t * kTK + half * kHK;
+        float sc[kHK];
+        if (key0 + kHK <= plen) {
 #pragma unroll
-        for (int k = 0; k < kTK; ++k) {
-          const int key = key0 + k;
-          const bool vis = all_prefix || (key < len && (key < plen || ((anc >> ((key - plen) & 63)) & 1ull)));
-          sc[k] = vis ? __uint_as_float(sr[k >> 5][k & 31]) * sl2 : -CUDART_INF_F;
-          tmax = fmaxf(tmax, sc[k]);
+          for (int k = 0; k < kHK; ++k) sc[k] = __uint_as_float(sr[k]) * sl2;
+        } else {
+#pragma unroll
+          for (int k = 0; k < kHK; ++k) {
+            const int key = key0 + k;
+            const bool vis = key < plen || (key < len && ((anc >> ((key - plen) & 63)) & 1ull));
+            sc[k] = vis ? __uint_as_float(sr[k]) * sl2 : -CUDART_INF_F;
+          }
         }
+        float mx[4] = {sc[0], sc[1], sc[2], sc[3]};
+#pragma unroll
+        for (int k = 4; k < kHK; ++k) mx[k & 3] = fmaxf(mx[k & 3], sc[k]);
+        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+
         const bool need = tmax > m_used + kRescaleLog2;
         if (__any_sync(0xffffffffu, need)) {
           const float m_new = need ? tmax : m_used;
@@ -317,11 +331,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
               for (int c = 0; c < D / 32; ++c) {
                 uint32_t o[32];
-                tc::tmem_ld32(lane_addr + C::kTmemO + c * 32, o);
+                tc::tmem_ld32(lane_addr + o_col + c * 32, o);
                 tc::tmem_wait_ld();
 #pragma unroll
                 for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
-                tc::tmem_st32(lane_addr + C::kTmemO + c * 32, o);
+                tc::tmem_st32(lane_addr + o_col + c * 32, o);
               }
               tc::tmem_wait_st();
             }
@@ -329,30 +343,32 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_used = m_new;
         }
         const float m_eff = m_used == -CUDART_INF_F ? 0.f : m_used;
-        uint32_t pk[kTK / 2];
-        float lsum = 0.f;
+        uint32_t pk[kHK / 2];
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int k = 0; k < kTK / 2; ++k) {
+        for (int k = 0; k < kHK / 2; ++k) {
           const float p0 = fast_exp2(sc[2 * k] - m_eff);
           const float p1 = fast_exp2(sc[2 * k + 1] - m_eff);
-          lsum += p0 + p1;
+          ls[k & 3] += p0 + p1;
           pk[k] = pack_bf16x2(p0, p1);
         }
-        l += lsum;
+        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
 
         if (!dead) dead = !warp_wait(&bars[B_PFREE + (j & 1)], ((j >> 1) & 1) ^ 1, abort_flag, p.status);
         {
           unsigned char* prow = base + C::off_P + (j & 1) * C::kPBytes + (row >> 3) * 1024 + (row & 7) * 128;
 #pragma unroll
-          for (int c = 0; c < 8; ++c)
-            *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) =
+          for (int c = 0; c < 4; ++c) {
+            const int chunk = half * 4 + c;  // 8 keys per 16-byte chunk
+            *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) =
                 make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+          }
         }
-        const int vrows = len - key0;
+        const int vrows = len - t * kTK;
         if (vrows < kTK) {  // last tile of the slab: clear V rows past its end
           const int st = j % kStages;
           if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (j / kStages) & 1, abort_flag, p.status);
-          for (int idx = row; idx < (kTK - vrows) * C::kHalves; idx += kSoft) {
+          for (int idx = sid; idx < (kTK - vrows) * C::kHalves; idx += kSoftWarps * 32) {
             const int r = vrows + idx / C::kHalves, hd = idx % C::kHalves;
             uint4* dst = reinterpret_cast<uint4*>(base + C::off_V + st * C::kKVTile + hd * C::kKVHalf + r * 128);
 #pragma unroll
@@ -365,36 +381,59 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bars[B_PFULL + (j & 1)]);
       }
 
-      // ---- segment epilogue: O / l, or a split partial
-      const int jl = i - 1;
-      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
-      const bool single = s.c_first == s.c_last;
-      const int bh = s.b * p.H + s.h;
-      float* dst = single ? p.out + (((size_t)s.b * n + row) * p.H + s.h) * D
-                          : partial_slot(p.partials, blockIdx.x + bh, n, D) + (size_t)row * (D + 2);
-      if (!dead) {
-        tc::fence_after_sync();
-        const float inv = single ? 1.f / l : 1.f;
+      // ---- segment epilogue: merge the two key halves, then O / l or a split partial
+      if (half == 1) ml[row] = make_float2(m_used, l);
+      softmax_sync();
+      if (half == 0) {
+        const int jl = i - 1;
+        if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+        const float2 other = ml[row];
+        const float M = fmaxf(m_used, other.x);
+        const float f0 = m_used == -CUDART_INF_F ? 0.f : fast_exp2(m_used - M);
+        const float f1 = other.x == -CUDART_INF_F ? 0.f : fast_exp2(other.x - M);
+        const float L = l * f0 + other.y * f1;
+        const bool single = s.c_first == s.c_last;
+        const int bh = s.b * p.H + s.h;
+        float* dst = single ? p.out + (((size_t)s.b * n + (valid ? qi : 0)) * p.H + s.h) * D
+                            : partial_slot(p.partials, blockIdx.x + bh, n, D) + (size_t)(valid ? qi : 0) * (D + 2);
+        if (!dead) {
+          tc::fence_after_sync();
+          const float g0 = single ? f0 / L : f0;
+          const float g1 = single ? f1 / L : f1;
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t o[32];
-          tc::tmem_ld32(lane_addr + C::kTmemO + c * 32, o);
-          tc::tmem_wait_ld();
-          if (row < n) {
-            float* d = dst + (single ? 0 : 2) + c * 32;
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t a[32], b[32];
+            tc::tmem_ld32(lane_addr + C::kTmemO + c * 32, a);
+            tc::tmem_ld32(lane_addr + C::kTmemO + D + c * 32, b);
+            tc::tmem_wait_ld();
+            if (valid) {
+              float4* d4 = reinterpret_cast<float4*>(dst + (single ? 0 : 2) + c * 32);
 #pragma unroll
-            for (int k = 0; k < 32; ++k) d[k] = __uint_as_float(o[k]) * inv;
+              for (int k = 0; k < 8; ++k) {
+                float4 v;
+                v.x = __uint_as_float(a[4 * k]) * g0 + __uint_as_float(b[4 * k]) * g1;
+                v.y = __uint_as_float(a[4 * k + 1]) * g0 + __uint_as_float(b[4 * k + 1]) * g1;
+                v.z = __uint_as_float(a[4 * k + 2]) * g0 + __uint_as_float(b[4 * k + 2]) * g1;
+                v.w = __uint_as_float(a[4 * k + 3]) * g0 + __uint_as_float(b[4 * k + 3]) * g1;
+                if (single) d4[k] = v;
+                else {  // partial rows are (D + 2) floats: only 8-byte aligned
+                  float2* d2 = reinterpret_cast<float2*>(d4 + k);
+                  d2[0] = make_float2(v.x, v.y);
+                  d2[1] = make_float2(v.z, v.w);
+                }
+              }
+            }
+          }
+          if (!single && valid) {
+            dst[0] = M;
+            dst[1] = L;
           }
         }
-        if (!single && row < n) {
-          dst[0] = m_used;
-          dst[1] = l;
-        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_OFREE]);
+        if (!single) combine_if_last(s, p.B, p.H, n, D, p.partials, p.counters, p.out, threadIdx.x, 128, last_flag);
       }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars[B_OFREE]);
-      if (!single) combine_if_last(s, p.B, p.H, n, D, p.partials, p.counters, p.out, row, kSoft, last_flag);
       g = s.g_end;
     }
   }
@@ -404,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == kMmaWarp) {
     tc::fence_after_sync();
-    tc::tmem_dealloc(tmem, kTmemCols);
+    tc::tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 
