@@ -35,7 +35,6 @@ constexpr int kThreads = (kNW + 1) * 32;
 
 template <typename T, int D>
 struct CrossCfg {
-  static constexpr int E = D / 32;                  // elements per lane
   static constexpr int kTile = kTK * D * (int)sizeof(T);
   static constexpr int kFit = (192 * 1024) / (2 * kTile * kNW);
   static constexpr int SW = kFit > 3 ? 3 : (kFit < 1 ? 1 : kFit);   // stages per consumer warp
@@ -68,7 +67,7 @@ struct CrossParams {
 template <typename T, int D>
 __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossParams p) {
   using C = CrossCfg<T, D>;
-  constexpr int E = C::E;
+  using G = GroupMap<T, D>;
   constexpr int NS = C::NS;
   extern __shared__ __align__(1024) unsigned char smem[];
   T* sK = reinterpret_cast<T*>(smem + C::off_K);
@@ -143,6 +142,7 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
   // -------------------------------------------------------------- consumers
   const int ctid = threadIdx.x;
   constexpr int kCT = kNW * 32;
+  const int sub = lane & 7, g4 = (lane >> 3) * 4;  // lane group g takes keys 4g..4g+3 of each tile
   const float sl2 = p.scale_log2;
   int i_base = 0;
   for (long long g = g_begin; g < g_end;) {
@@ -150,14 +150,18 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
     const int ntile = s.t1 - s.t0;
     const int len = bt.len[s.b];
 
-    float q[E];
-    load_row_chunk<T, E>(static_cast<const T*>(p.q) + ((size_t)s.b * p.H + s.h) * D + lane * E, q);
+    // q chunks of this lane (raw; the scale is applied to the finished score)
+    uint4 qc[G::kNC];
+    {
+      const unsigned char* qrow =
+          reinterpret_cast<const unsigned char*>(static_cast<const T*>(p.q) + ((size_t)s.b * p.H + s.h) * D);
 #pragma unroll
-    for (int e = 0; e < E; ++e) q[e] *= sl2;
-
-    float m = -CUDART_INF_F, l = 0.f, o[E];
+      for (int m = 0; m < G::kNC; ++m) qc[m] = *reinterpret_cast<const uint4*>(qrow + (sub + 8 * m) * 16);
+    }
+    float m = -CUDART_INF_F, l = 0.f;
+    uint64_t o2[G::kPairs];
 #pragma unroll
-    for (int e = 0; e < E; ++e) o[e] = 0.f;
+    for (int e = 0; e < G::kPairs; ++e) o2[e] = 0ull;
 
     const int first = i_base + (((warp - i_base) % kNW) + kNW) % kNW;
     for (int i = first; i < i_base + ntile; i += kNW) {
@@ -166,48 +170,69 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
       if (!mbar_wait(&full[st], (r / C::SW) & 1, abort_flag, p.status)) break;
       const int t = s.t0 + (i - i_base);
       const int rows = min(kTK, len - t * kTK);
-      const T* Kt = sK + (size_t)st * kTK * D + lane * E;
-      const T* Vt = sV + (size_t)st * kTK * D + lane * E;
+      const unsigned char* Kb = reinterpret_cast<const unsigned char*>(sK + (size_t)st * kTK * D);
+      const unsigned char* Vb = reinterpret_cast<const unsigned char*>(sV + (size_t)st * kTK * D);
 
-      float part[kTK];
+      // Copy this lane's K and V chunks of the tile to registers and hand the
+      // stage back at once, so the ring stays in flight while the warp computes.
+      uint4 kr[4][G::kNC], vr[4][G::kNC];
 #pragma unroll
-      for (int k = 0; k < kTK; ++k) {
-        float kf[E];
-        load_row_chunk<T, E>(Kt + k * D, kf);
-        float acc = 0.f;
+      for (int kk = 0; kk < 4; ++kk)
 #pragma unroll
-        for (int e = 0; e < E; ++e) acc = fmaf(q[e], kf[e], acc);
-        part[k] = acc;
+        for (int mm = 0; mm < G::kNC; ++mm) {
+          kr[kk][mm] = *reinterpret_cast<const uint4*>(Kb + (g4 + kk) * G::kRowBytes + (sub + 8 * mm) * 16);
+          vr[kk][mm] = *reinterpret_cast<const uint4*>(Vb + (g4 + kk) * G::kRowBytes + (sub + 8 * mm) * 16);
+        }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+
+      // partial scores of this group's 4 keys over this lane's dims
+      float part[4];
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        float acc[2] = {0.f, 0.f};
+#pragma unroll
+        for (int mm = 0; mm < G::kNC; ++mm) dot_chunk<T>(qc[mm], kr[kk][mm], acc);
+        part[kk] = acc[0] + acc[1];
       }
-      float sc = transpose_reduce16(part, lane);  // score of key lane / 2
+      float sc = group8_reduce4(part, lane) * sl2;  // score of key lane / 2 of the tile
       if ((lane >> 1) >= rows) sc = -CUDART_INF_F;
       const float m_new = fmaxf(m, warp_max(sc));
       const float corr = fast_exp2(m - m_new);
       const float pe = fast_exp2(sc - m_new);
       l = l * corr + ((lane & 1) ? 0.f : pe);  // each key is held by two lanes: count it once
+      const uint64_t corr2 = f2pack(corr, corr);
 #pragma unroll
-      for (int e = 0; e < E; ++e) o[e] *= corr;
+      for (int e = 0; e < G::kPairs; ++e) o2[e] = f2mul(o2[e], corr2);
 #pragma unroll
-      for (int k = 0; k < kTK; ++k) {
-        if (k < rows) {
-          const float pk = __shfl_sync(0xffffffffu, pe, 2 * k);
-          float vf[E];
-          load_row_chunk<T, E>(Vt + k * D, vf);
+      for (int kk = 0; kk < 4; ++kk) {
+        const float pk = __shfl_sync(0xffffffffu, pe, (lane & ~7) + 2 * kk);
+        if (g4 + kk < rows) {  // rows past the slab end hold stale data (even NaN): skip them
+          const uint64_t p2 = f2pack(pk, pk);
 #pragma unroll
-          for (int e = 0; e < E; ++e) o[e] = fmaf(pk, vf[e], o[e]);
+          for (int mm = 0; mm < G::kNC; ++mm) axpy_chunk<T>(p2, vr[kk][mm], o2 + mm * G::kPairsPerChunk);
         }
       }
       m = m_new;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[st]);
     }
 
-    // ---- merge the warps' partial results of this segment
+    // ---- merge: lane groups within the warp, then the warps of the CTA
     l = warp_sum(l);
     float* my = scratch + warp * (D + 2);
     if (lane == 0) { my[0] = m; my[1] = l; }
 #pragma unroll
-    for (int e = 0; e < E; ++e) my[2 + lane * E + e] = o[e];
+    for (int e = 0; e < G::kPairs; ++e) {
+      float2 v = f2unpack(o2[e]);
+      v.x += __shfl_xor_sync(0xffffffffu, v.x, 8);
+      v.y += __shfl_xor_sync(0xffffffffu, v.y, 8);
+      v.x += __shfl_xor_sync(0xffffffffu, v.x, 16);
+      v.y += __shfl_xor_sync(0xffffffffu, v.y, 16);
+      if (lane < 8) {
+        const int d = (sub + 8 * (e / G::kPairsPerChunk)) * G::kChunkElems + 2 * (e % G::kPairsPerChunk);
+        my[2 + d] = v.x;
+        my[3 + d] = v.y;
+      }
+    }
     consumer_sync(kCT);
 
     float M = -CUDART_INF_F;

@@ -6,26 +6,31 @@
 // At n = 26..64 queries the verification does n flops per KV byte, beyond
 // what CUDA-core FMA can sustain at HBM speed, so both products run on the
 // tensor cores while the KV stream stays the bound:
-//   S = Q K^T   : M = 128 (query rows, zero-padded), N = 64 keys, K = D
-//   O += P V    : M = 128, N = D, K = 32 keys, once per key half
+//   S = Q K^T   : M = 64 (query rows, zero-padded), N = 64 keys, K = D
+//   O += P V    : M = 64, N = D, K = 32 keys, once per key half
 // Operands sit in shared memory in the 128-byte-swizzled K-major layout
 // (Q, K, P) or M/N-major layout (V); accumulators live in tensor memory
-// (TMEM): two S buffers of 64 columns and one O accumulator of D columns for
+// (TMEM): four S buffers of 64 columns and one O accumulator of D columns for
 // each key half.
 //
-// Roles (320 threads, persistent grid of one CTA per SM, split-KV partition
+// Roles (384 threads, persistent grid of one CTA per SM, split-KV partition
 // shared with the other attention kernels):
-//   warps 0-7  softmax.  Warp w reads TMEM lane quarter w % 4 (32 query
-//              rows) and key half w / 4 (32 of the tile's 64 keys).  Each
+//   warps 0-7  softmax.  An M = 64 accumulator keeps rows 16q..16q+15 in
+//              TMEM lanes 32q..32q+15; warp w reads lane quarter q = w % 4
+//              with the 16x64b shape (two threads per row, even and odd
+//              columns) and key half w / 4 (32 of the tile's 64 keys).  Each
 //              (row, key half) keeps its own running max and sum and its own
 //              O accumulator, so no values cross warps inside the key loop;
 //              the halves are merged once per segment.  Query i sits in row
-//              (i % 4) * 32 + i / 4, which spreads any tree over all four
-//              lane quarters (all four SM sub-partitions).
+//              (i % 4) * 16 + i / 4, which spreads any tree over all four lane
+//              quarters (all four SM sub-partitions).
 //   warp 8     producer: lane 0 loads K tiles, lane 1 V tiles, with 2-D TMA
 //              (64 keys x 64 head dims per box, 128-byte swizzle).
-//   warp 9     MMA: allocates TMEM; one thread issues S(j+1) before PV(j) so
-//              the softmax of one tile overlaps the P.V product of the last.
+//   warps 9-11 MMA issue.  A tcgen05.mma keeps its issuing thread busy for
+//              ~150 cycles whatever its shape, so one thread cannot feed a
+//              64-key tile (8 S + 4 P.V instructions) at HBM speed: warp 9
+//              issues S for even tiles, warp 10 S for odd tiles, warp 11 all
+//              P.V products.  Warp 9 also owns the TMEM allocation.
 //
 // Online softmax in the log2 domain with a lazy reference max: the max used
 // for the exponent only moves when a tile's max exceeds it by more than 8
@@ -49,38 +54,46 @@ namespace {
 
 constexpr int kTK = 64;          // keys per tile
 constexpr int kHK = 32;          // keys per key half
-constexpr int kM = 128;          // MMA rows
-constexpr int kStages = 4;       // K/V stages
+constexpr int kM = 64;           // MMA rows (tree queries, zero-padded)
+constexpr int kMaxStages = 8;    // K/V stages (the launch picks as many as fit)
+constexpr int kSBuf = 4;         // S buffers in TMEM (two per S issuer)
 constexpr int kSoftWarps = 8;
 constexpr int kProdWarp = 8;
-constexpr int kMmaWarp = 9;
-constexpr int kThreads = 320;
+constexpr int kMmaWarp = 9;      // warps 9, 10: S issuers; warp 11: P.V issuer
+constexpr int kThreads = 384;
 constexpr float kRescaleLog2 = 8.0f;
 
 // barrier slots
-constexpr int B_KFULL = 0, B_VFULL = 4, B_KEMPTY = 8, B_VEMPTY = 12, B_SFULL = 16, B_SFREE = 18, B_PFULL = 20,
-              B_PFREE = 22, B_ODONE = 24, B_OFREE = 26, B_QFULL = 27, B_MDONE = 28, kNumBars = 29;
+// ODONE has four slots (tile mod 4): the softmax waits on it only now and
+// then, and four slots keep every such wait within one phase of the barrier.
+// QFULL has two slots (segment parity): an S issuer waits only for segments
+// in which it has a tile, and each issuer has a tile in every two consecutive
+// segments, so no slot runs two phases ahead of a waiter.
+constexpr int B_KFULL = 0, B_VFULL = 8, B_KEMPTY = 16, B_VEMPTY = 24, B_SFULL = 32, B_SFREE = 36, B_PFULL = 40,
+              B_PFREE = 42, B_ODONE = 44, B_OFREE = 48, B_QFULL = 49, B_MDONE = 51, kNumBars = 54;
 
 template <int D>
 struct TcCfg {
   static constexpr int kHalves = D / 64;              // 128-byte swizzle atoms across the head dim
-  static constexpr uint32_t kQHalf = kM * 128;        // 128 rows x 128 B
+  static constexpr uint32_t kQHalf = kM * 128;        // 64 rows x 128 B
   static constexpr uint32_t kQBytes = kHalves * kQHalf;
-  static constexpr uint32_t kPBytes = kM * kTK * 2;   // 128 rows x 64 keys bf16
+  static constexpr uint32_t kPBytes = kM * kTK * 2;   // 64 rows x 64 keys bf16
   static constexpr uint32_t kKVHalf = kTK * 128;      // 64 keys x 128 B
   static constexpr uint32_t kKVTile = kHalves * kKVHalf;
   static constexpr uint32_t off_Q = 0;
   static constexpr uint32_t off_P = off_Q + kQBytes;
   static constexpr uint32_t off_K = off_P + 2 * kPBytes;
-  static constexpr uint32_t off_V = off_K + kStages * kKVTile;
-  static constexpr uint32_t off_bar = off_V + kStages * kKVTile;
-  static constexpr uint32_t off_ml = off_bar + 256;                // [128] (max, sum) of key half 1
-  static constexpr uint32_t off_misc = off_ml + kM * 8;
-  static constexpr uint32_t off_tab = off_misc + 32;
-  static constexpr uint32_t kTmemO = 2 * kTK;                      // S buffers at columns 0 and 64
+  // then ns K stages, ns V stages, barriers, (max, sum) of key half 1, misc, batch table
+  static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKVTile; }
+  static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKVTile; }
+  static __host__ __device__ uint32_t off_ml(int ns) { return off_bar(ns) + 512; }
+  static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + kM * 8; }
+  static __host__ __device__ uint32_t off_tab(int ns) { return off_misc(ns) + 32; }
+  static constexpr uint32_t kTmemO = kSBuf * kTK;                  // S buffers at columns 0, 64, 128, 192
   static constexpr uint32_t kTmemCols = kTmemO + 2 * D <= 256 ? 256 : 512;
-  static_assert(kNumBars * 8 <= 256, "barrier area");
-  static size_t smem_bytes(int B) { return 1024 + off_tab + (size_t)(B + 1) * 8 + (size_t)3 * B * 4; }
+  static_assert(kTmemO + 2 * D <= 512, "TMEM columns");
+  static_assert(kNumBars * 8 <= 512, "barrier area");
+  static size_t smem_bytes(int B, int ns) { return 1024 + off_tab(ns) + (size_t)(B + 1) * 8 + (size_t)3 * B * 4; }
 };
 
 struct TcParams {
@@ -92,6 +105,7 @@ struct TcParams {
   unsigned* counters;
   float* partials;
   int B, H, S_cap, max_kv_len, n;
+  int ns;  // K/V stages
   float scale_log2;
 };
 
@@ -121,13 +135,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   using C = TcCfg<D>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar);
-  float2* ml = reinterpret_cast<float2*>(base + C::off_ml);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc + 4);
-  volatile int* last_flag = reinterpret_cast<volatile int*>(base + C::off_misc + 8);
+  const int ns = p.ns;
+  const uint32_t off_V = C::off_V(ns);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(ns));
+  float2* ml = reinterpret_cast<float2*>(base + C::off_ml(ns));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
+  volatile int* last_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 8);
   BatchTiles bt;
-  bt.start = reinterpret_cast<long long*>(base + C::off_tab);
+  bt.start = reinterpret_cast<long long*>(base + C::off_tab(ns));
   bt.len = reinterpret_cast<int*>(bt.start + p.B + 1);
   bt.ntiles = bt.len + p.B;
   bt.plen = bt.ntiles + p.B;
@@ -137,8 +153,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int b = 0; b < kNumBars; ++b) {
       uint32_t cnt = 1;
-      if (b == B_SFREE || b == B_SFREE + 1 || b == B_PFULL || b == B_PFULL + 1) cnt = kSoftWarps;
-      if (b == B_OFREE || b == B_QFULL) cnt = 4;  // the key-half-0 warps
+      if ((b >= B_SFREE && b < B_SFREE + kSBuf) || b == B_PFULL || b == B_PFULL + 1) cnt = kSoftWarps;
+      if (b == B_OFREE || b == B_QFULL || b == B_QFULL + 1) cnt = 4;  // the key-half-0 warps
       mbar_init(&bars[b], cnt);
     }
     *abort_flag = 0;
@@ -159,48 +175,107 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kProdWarp) {
     // ------------------------------------------------------------ producer
-    if (lane < 2) {  // lane 0: K tiles, lane 1: V tiles
-      const CUtensorMap* map = lane == 0 ? &tmK : &tmV;
-      uint64_t* full = &bars[lane == 0 ? B_KFULL : B_VFULL];
-      uint64_t* empty = &bars[lane == 0 ? B_KEMPTY : B_VEMPTY];
-      const uint32_t dst0 = lane == 0 ? C::off_K : C::off_V;
-      tc::prefetch_tmap(map);
+    // One thread feeds both rings without blocking on either: K slots free up
+    // when S is done, V slots only when P.V is done, and a blocking wait on
+    // one ring would hold back the other.
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmK);
+      tc::prefetch_tmap(&tmV);
       const uint64_t pol = policy_evict_first();
-      int i = 0;
-      bool ok = true;
-      for (long long g = g_begin; g < g_end && ok;) {
-        const Segment s = locate(bt, P, p.B, g, g_end);
-        const int slab_row = (s.b * p.H + s.h) * p.S_cap;
-        for (int t = s.t0; t < s.t1; ++t, ++i) {
-          const int st = i % kStages;
-          if (!mbar_wait(&empty[st], ((i / kStages) & 1) ^ 1, abort_flag, p.status)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[st], C::kKVTile);
-          for (int hd = 0; hd < C::kHalves; ++hd)
-            tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, slab_row + t * kTK,
-                            &full[st], pol);
+      struct Cursor {  // next tile to load: CTA-local index i, segment s, tile t
+        int i, t;
+        long long g;
+        Segment s;
+      };
+      auto start_seg = [&](Cursor& c) {
+        if (c.g < g_end) {
+          c.s = locate(bt, P, p.B, c.g, g_end);
+          c.t = c.s.t0;
         }
-        g = s.g_end;
+      };
+      auto issue = [&](Cursor& c, const CUtensorMap* map, uint64_t* full, uint32_t dst0) {
+        const int st = c.i % ns;
+        mbar_arrive_expect_tx(&full[st], C::kKVTile);
+        const int row = (c.s.b * p.H + c.s.h) * p.S_cap + c.t * kTK;
+        for (int hd = 0; hd < C::kHalves; ++hd)
+          tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, row, &full[st], pol);
+        ++c.i;
+        if (++c.t == c.s.t1) {
+          c.g = c.s.g_end;
+          start_seg(c);
+        }
+      };
+      Cursor ck, cv;
+      ck.i = cv.i = 0;
+      ck.g = cv.g = g_begin;
+      start_seg(ck);
+      start_seg(cv);
+      const int total = (int)(g_end - g_begin);
+      uint64_t t_last = global_timer_ns();
+      int spins = 0, seen = 0;
+      while (ck.i < total || cv.i < total) {
+        bool progressed = false;
+        if (ck.i < total && mbar_test_wait(&bars[B_KEMPTY + ck.i % ns], ((ck.i / ns) & 1) ^ 1)) {
+          issue(ck, &tmK, &bars[B_KFULL], C::off_K);
+          progressed = true;
+        }
+        if (cv.i < total && mbar_test_wait(&bars[B_VEMPTY + cv.i % ns], ((cv.i / ns) & 1) ^ 1)) {
+          issue(cv, &tmV, &bars[B_VFULL], off_V);
+          progressed = true;
+        }
+        if (progressed || ++spins < 64) continue;
+        spins = 0;  // every 64 idle polls: check for an abort or a stall of more than kWaitLimitNs
+        const uint64_t now = global_timer_ns();
+        if (ck.i + cv.i != seen) {
+          seen = ck.i + cv.i;
+          t_last = now;
+        }
+        if (*abort_flag) break;
+        if (now - t_last > kWaitLimitNs) {
+          *abort_flag = 1;
+          record_status(p.status, kStatusTimeout);
+          break;
+        }
       }
-      if (!ok) {  // let issued loads land before the CTA exits
-        for (int j = (i > kStages ? i - kStages : 0); j < i; ++j) mbar_drain(&full[j % kStages], (j / kStages) & 1);
+      if (ck.i < total || cv.i < total) {  // aborted: let issued loads land before the CTA exits
+        for (int j = (ck.i > ns ? ck.i - ns : 0); j < ck.i; ++j) mbar_drain(&bars[B_KFULL + j % ns], (j / ns) & 1);
+        for (int j = (cv.i > ns ? cv.i - ns : 0); j < cv.i; ++j) mbar_drain(&bars[B_VFULL + j % ns], (j / ns) & 1);
       }
     }
-  } else if (warp == kMmaWarp) {
-    // ----------------------------------------------------------------- MMA
+  } else if (warp >= kMmaWarp) {
+    // ----------------------------------------------------------- MMA issue
+    const int role = warp - kMmaWarp;  // 0, 1: S of tiles with j % 2 == role; 2: P.V
     if (lane == 0) {
       constexpr uint32_t idS = tc::idesc_bf16_f32(kM, kTK, false, false);
       constexpr uint32_t idO = tc::idesc_bf16_f32(kM, D, false, true);
       const uint32_t sQ = smem_u32(base + C::off_Q), sP = smem_u32(base + C::off_P);
-      const uint32_t sK = smem_u32(base + C::off_K), sV = smem_u32(base + C::off_V);
+      const uint32_t sK = smem_u32(base + C::off_K), sV = smem_u32(base + off_V);
       int i = 0, seg = 0;
       bool ok = true;
+      // S(j) = Q K(j)^T into S buffer j % kSBuf
+      auto issue_s = [&](int j) -> bool {
+        if (!mbar_wait(&bars[B_KFULL + j % ns], (j / ns) & 1, abort_flag, p.status) ||
+            !mbar_wait(&bars[B_SFREE + j % kSBuf], ((j / kSBuf) & 1) ^ 1, abort_flag, p.status))
+          return false;
+        tc::fence_after_sync();
+        const uint32_t kb = sK + (j % ns) * C::kKVTile;
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint64_t a = tc::sw128_desc(sQ + (ks / 4) * C::kQHalf + (ks % 4) * 32, 16, 1024);
+          const uint64_t bdesc = tc::sw128_desc(kb + (ks / 4) * C::kKVHalf + (ks % 4) * 32, 16, 1024);
+          tc::mma_bf16(tmem + (j % kSBuf) * kTK, a, bdesc, idS, ks > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(&bars[B_SFULL + j % kSBuf]);
+        tc::mma_commit(&bars[B_KEMPTY + j % ns]);
+        return true;
+      };
       // O_h += P[:, 32h .. 32h+31] V[32h .. 32h+31, :] for key halves h = 0, 1
       auto issue_pv = [&](int jj, bool first_in_seg) -> bool {
         if (!mbar_wait(&bars[B_PFULL + (jj & 1)], (jj >> 1) & 1, abort_flag, p.status)) return false;
-        if (!mbar_wait(&bars[B_VFULL + jj % kStages], (jj / kStages) & 1, abort_flag, p.status)) return false;
+        if (!mbar_wait(&bars[B_VFULL + jj % ns], (jj / ns) & 1, abort_flag, p.status)) return false;
         if (first_in_seg && seg > 0 && !mbar_wait(&bars[B_OFREE], (seg - 1) & 1, abort_flag, p.status)) return false;
         tc::fence_after_sync();
-        const uint32_t vb = sV + (jj % kStages) * C::kKVTile;
+        const uint32_t vb = sV + (jj % ns) * C::kKVTile;
         const uint32_t pb = sP + (jj & 1) * C::kPBytes;
 #pragma unroll
         for (int ks = 0; ks < kTK / 16; ++ks) {
@@ -210,71 +285,70 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc::mma_bf16(tmem + C::kTmemO + h * D, a, bdesc, idO, (first_in_seg && (ks & 1) == 0) ? 0u : 1u);
         }
         tc::mma_commit(&bars[B_PFREE + (jj & 1)]);
-        tc::mma_commit(&bars[B_VEMPTY + jj % kStages]);
-        tc::mma_commit(&bars[B_ODONE + (jj & 1)]);
+        tc::mma_commit(&bars[B_VEMPTY + jj % ns]);
+        tc::mma_commit(&bars[B_ODONE + (jj & 3)]);
         return true;
       };
       for (long long g = g_begin; g < g_end && ok;) {
         const Segment s = locate(bt, P, p.B, g, g_end);
-        if (!mbar_wait(&bars[B_QFULL], seg & 1, abort_flag, p.status)) { ok = false; break; }
-        for (int t = s.t0; t < s.t1; ++t, ++i) {
-          const int j = i;
-          if (!mbar_wait(&bars[B_KFULL + j % kStages], (j / kStages) & 1, abort_flag, p.status) ||
-              !mbar_wait(&bars[B_SFREE + (j & 1)], ((j >> 1) & 1) ^ 1, abort_flag, p.status)) {
+        if (role < 2) {
+          // S of the tiles j with j % 2 == role; Q of the segment must be in place first
+          const int ntile = s.t1 - s.t0;
+          const bool mine = ntile > 1 || (i & 1) == role;
+          if (mine && !mbar_wait(&bars[B_QFULL + (seg & 1)], (seg >> 1) & 1, abort_flag, p.status)) {
             ok = false;
             break;
           }
-          tc::fence_after_sync();
-          const uint32_t kb = sK + (j % kStages) * C::kKVTile;
-#pragma unroll
-          for (int ks = 0; ks < D / 16; ++ks) {
-            const uint64_t a = tc::sw128_desc(sQ + (ks / 4) * C::kQHalf + (ks % 4) * 32, 16, 1024);
-            const uint64_t bdesc = tc::sw128_desc(kb + (ks / 4) * C::kKVHalf + (ks % 4) * 32, 16, 1024);
-            tc::mma_bf16(tmem + (j & 1) * kTK, a, bdesc, idS, ks > 0 ? 1u : 0u);
-          }
-          tc::mma_commit(&bars[B_SFULL + (j & 1)]);
-          tc::mma_commit(&bars[B_KEMPTY + j % kStages]);
-          if (t > s.t0 && !issue_pv(j - 1, t - 1 == s.t0)) { ok = false; break; }
+          for (int t = s.t0; t < s.t1 && ok; ++t, ++i)
+            if ((i & 1) == role) ok = issue_s(i);
+        } else {
+          for (int t = s.t0; t < s.t1 && ok; ++t, ++i) ok = issue_pv(i, t == s.t0);
         }
-        if (ok && !issue_pv(i - 1, s.t1 - 1 == s.t0)) ok = false;
         ++seg;
         g = s.g_end;
       }
-      tc::mma_commit(&bars[B_MDONE]);  // every MMA finished before TMEM is released
-      mbar_drain(&bars[B_MDONE], 0);
+      tc::mma_commit(&bars[B_MDONE + role]);  // every MMA finished before TMEM is released
+      mbar_drain(&bars[B_MDONE + role], 0);
     }
   } else {
     // ------------------------------------------------------------- softmax
+    // Warp w reads lane quarter q = w % 4 (MMA rows 16q..16q+15) and key half
+    // w / 4 with the 16x64b TMEM shape: lane pair (t, t^2) shares one row,
+    // thread t takes the row's even or odd columns (cpar), 16 of the 32 keys.
     const int quarter = warp & 3, half = warp >> 2;
-    const int row = quarter * 32 + lane;       // TMEM lane = MMA row
-    const int qi = lane * 4 + quarter;         // the tree query in this row
+    const int rr = (lane >> 2) + 8 * (lane & 1);  // row within the quarter
+    const int cpar = (lane >> 1) & 1;             // column parity of this thread
+    const int row = quarter * 16 + rr;            // MMA row
+    const int qi = rr * 4 + quarter;              // the tree query in this row
     const bool valid = qi < n;
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t o_col = C::kTmemO + half * D;
-    const int sid = threadIdx.x;               // 0..255 among the softmax threads
+    const int sid = threadIdx.x;                  // 0..255 among the softmax threads
     const float sl2 = p.scale_log2;
     bool dead = false;
-    int i = 0;
-    for (long long g = g_begin; g < g_end;) {
+    int i = 0, seg = 0;
+    for (long long g = g_begin; g < g_end; ++seg) {
       const Segment s = locate(bt, P, p.B, g, g_end);
       const int plen = bt.plen[s.b], len = bt.len[s.b];
 
       if (half == 0) {
-        // this segment's queries into the swizzled Q tile (padding rows are zero)
+        // this segment's queries into the swizzled Q tile (padding rows are zero);
+        // the two threads of a row write chunks 0-3 and 4-7 of each 128-byte atom
         unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
         const uint4* src =
             reinterpret_cast<const uint4*>(p.q + (((size_t)s.b * n + (valid ? qi : 0)) * p.H + s.h) * D);
 #pragma unroll
         for (int hd = 0; hd < C::kHalves; ++hd)
 #pragma unroll
-          for (int c = 0; c < 8; ++c) {
+          for (int cc = 0; cc < 4; ++cc) {
+            const int c = cpar * 4 + cc;
             uint4 v = make_uint4(0u, 0u, 0u, 0u);
             if (valid) v = src[hd * 8 + c];
             *reinterpret_cast<uint4*>(qrow + hd * C::kQHalf + ((c ^ (row & 7)) << 4)) = v;
           }
         tc::fence_async_smem();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars[B_QFULL]);
+        if (lane == 0) mbar_arrive(&bars[B_QFULL + (seg & 1)]);
       }
       uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
       if (valid) {
@@ -286,38 +360,39 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
 
-      float m_used = -CUDART_INF_F, l = 0.f;
+      float m_used = -CUDART_INF_F, l = 0.f;  // l: this thread's share of the row sum
       for (int t = s.t0; t < s.t1; ++t, ++i) {
         const int j = i;
-        uint32_t sr[32];
-        if (!dead) dead = !warp_wait(&bars[B_SFULL + (j & 1)], (j >> 1) & 1, abort_flag, p.status);
+        uint32_t sr[16];
+        if (!dead) dead = !warp_wait(&bars[B_SFULL + j % kSBuf], (j / kSBuf) & 1, abort_flag, p.status);
         if (!dead) {
           tc::fence_after_sync();
-          tc::tmem_ld32(lane_addr + (j & 1) * kTK + half * kHK, sr);
+          tc::tmem_ld16x64b_x16(lane_addr + (j % kSBuf) * kTK + half * kHK, sr);
           tc::tmem_wait_ld();
         }
         tc::fence_before_sync();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars[B_SFREE + (j & 1)]);
+        if (lane == 0) mbar_arrive(&bars[B_SFREE + j % kSBuf]);
 
-        // scores of this key half in the log2 domain, masked
-        const int key0 = t * kTK + half * kHK;
-        float sc[kHK];
-        if (key0 + kHK <= plen) {
+        // scores of keys key0 + 2k + cpar, k = 0..15, in the log2 domain, masked
+        const int key0 = t * kTK + half * kHK + cpar;
+        float sc[16];
+        if (t * kTK + half * kHK + kHK <= plen) {
 #pragma unroll
-          for (int k = 0; k < kHK; ++k) sc[k] = __uint_as_float(sr[k]) * sl2;
+          for (int k = 0; k < 16; ++k) sc[k] = __uint_as_float(sr[k]) * sl2;
         } else {
 #pragma unroll
-          for (int k = 0; k < kHK; ++k) {
-            const int key = key0 + k;
+          for (int k = 0; k < 16; ++k) {
+            const int key = key0 + 2 * k;
             const bool vis = key < plen || (key < len && ((anc >> ((key - plen) & 63)) & 1ull));
             sc[k] = vis ? __uint_as_float(sr[k]) * sl2 : -CUDART_INF_F;
           }
         }
         float mx[4] = {sc[0], sc[1], sc[2], sc[3]};
 #pragma unroll
-        for (int k = 4; k < kHK; ++k) mx[k & 3] = fmaxf(mx[k & 3], sc[k]);
-        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        for (int k = 4; k < 16; ++k) mx[k & 3] = fmaxf(mx[k & 3], sc[k]);
+        float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));  // the row's max over both threads
 
         const bool need = tmax > m_used + kRescaleLog2;
         if (__any_sync(0xffffffffu, need)) {
@@ -325,17 +400,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float f = need ? fast_exp2(m_used - m_new) : 1.f;
           l *= f;
           if (t > s.t0 && !dead) {  // O holds the P.V of earlier tiles of this segment
-            dead = !warp_wait(&bars[B_ODONE + ((j - 1) & 1)], ((j - 1) >> 1) & 1, abort_flag, p.status);
+            dead = !warp_wait(&bars[B_ODONE + ((j - 1) & 3)], ((j - 1) >> 2) & 1, abort_flag, p.status);
             if (!dead) {
               tc::fence_after_sync();
 #pragma unroll 1
               for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tc::tmem_ld32(lane_addr + o_col + c * 32, o);
+                uint32_t o[16];
+                tc::tmem_ld16x64b_x16(lane_addr + o_col + c * 32, o);
                 tc::tmem_wait_ld();
 #pragma unroll
-                for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
-                tc::tmem_st32(lane_addr + o_col + c * 32, o);
+                for (int k = 0; k < 16; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * f);
+                tc::tmem_st16x64b_x16(lane_addr + o_col + c * 32, o);
               }
               tc::tmem_wait_st();
             }
@@ -343,34 +418,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_used = m_new;
         }
         const float m_eff = m_used == -CUDART_INF_F ? 0.f : m_used;
-        uint32_t pk[kHK / 2];
+        float pv[16];
         float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int k = 0; k < kHK / 2; ++k) {
-          const float p0 = fast_exp2(sc[2 * k] - m_eff);
-          const float p1 = fast_exp2(sc[2 * k + 1] - m_eff);
-          ls[k & 3] += p0 + p1;
-          pk[k] = pack_bf16x2(p0, p1);
+        for (int k = 0; k < 16; ++k) {
+          pv[k] = fast_exp2(sc[k] - m_eff);
+          ls[k & 3] += pv[k];
         }
         l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        // bf16 pairs of consecutive keys: the even-column thread keeps keys 0..15
+        // of the half, the odd-column thread keys 16..31; swap the other halves
+        uint32_t pk[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const float send = cpar ? pv[k] : pv[8 + k];
+          const float recv = __shfl_xor_sync(0xffffffffu, send, 2);
+          pk[k] = cpar ? pack_bf16x2(recv, pv[8 + k]) : pack_bf16x2(pv[k], recv);
+        }
 
         if (!dead) dead = !warp_wait(&bars[B_PFREE + (j & 1)], ((j >> 1) & 1) ^ 1, abort_flag, p.status);
         {
           unsigned char* prow = base + C::off_P + (j & 1) * C::kPBytes + (row >> 3) * 1024 + (row & 7) * 128;
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const int chunk = half * 4 + c;  // 8 keys per 16-byte chunk
+          for (int c = 0; c < 2; ++c) {
+            const int chunk = half * 4 + cpar * 2 + c;  // 8 keys per 16-byte chunk
             *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) =
                 make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
           }
         }
         const int vrows = len - t * kTK;
         if (vrows < kTK) {  // last tile of the slab: clear V rows past its end
-          const int st = j % kStages;
-          if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (j / kStages) & 1, abort_flag, p.status);
+          const int st = j % ns;
+          if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (j / ns) & 1, abort_flag, p.status);
           for (int idx = sid; idx < (kTK - vrows) * C::kHalves; idx += kSoftWarps * 32) {
             const int r = vrows + idx / C::kHalves, hd = idx % C::kHalves;
-            uint4* dst = reinterpret_cast<uint4*>(base + C::off_V + st * C::kKVTile + hd * C::kKVHalf + r * 128);
+            uint4* dst = reinterpret_cast<uint4*>(base + off_V + st * C::kKVTile + hd * C::kKVHalf + r * 128);
 #pragma unroll
             for (int c = 0; c < 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
           }
@@ -382,11 +464,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
 
       // ---- segment epilogue: merge the two key halves, then O / l or a split partial
-      if (half == 1) ml[row] = make_float2(m_used, l);
+      l += __shfl_xor_sync(0xffffffffu, l, 2);  // the row's sum over both threads
+      if (half == 1 && cpar == 0) ml[row] = make_float2(m_used, l);
       softmax_sync();
       if (half == 0) {
         const int jl = i - 1;
-        if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+        if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 3)], (jl >> 2) & 1, abort_flag, p.status);
         const float2 other = ml[row];
         const float M = fmaxf(m_used, other.x);
         const float f0 = m_used == -CUDART_INF_F ? 0.f : fast_exp2(m_used - M);
@@ -395,38 +478,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool single = s.c_first == s.c_last;
         const int bh = s.b * p.H + s.h;
         float* dst = single ? p.out + (((size_t)s.b * n + (valid ? qi : 0)) * p.H + s.h) * D
-                            : partial_slot(p.partials, blockIdx.x + bh, n, D) + (size_t)(valid ? qi : 0) * (D + 2);
+                            : partial_slot(p.partials, blockIdx.x + bh, n, D) + (size_t)(valid ? qi : 0) * (D + 2) + 2;
         if (!dead) {
           tc::fence_after_sync();
           const float g0 = single ? f0 / L : f0;
           const float g1 = single ? f1 / L : f1;
 #pragma unroll 1
           for (int c = 0; c < D / 32; ++c) {
-            uint32_t a[32], b[32];
-            tc::tmem_ld32(lane_addr + C::kTmemO + c * 32, a);
-            tc::tmem_ld32(lane_addr + C::kTmemO + D + c * 32, b);
+            uint32_t a[16], b[16];
+            tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + c * 32, a);
+            tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + D + c * 32, b);
             tc::tmem_wait_ld();
             if (valid) {
-              float4* d4 = reinterpret_cast<float4*>(dst + (single ? 0 : 2) + c * 32);
 #pragma unroll
-              for (int k = 0; k < 8; ++k) {
-                float4 v;
-                v.x = __uint_as_float(a[4 * k]) * g0 + __uint_as_float(b[4 * k]) * g1;
-                v.y = __uint_as_float(a[4 * k + 1]) * g0 + __uint_as_float(b[4 * k + 1]) * g1;
-                v.z = __uint_as_float(a[4 * k + 2]) * g0 + __uint_as_float(b[4 * k + 2]) * g1;
-                v.w = __uint_as_float(a[4 * k + 3]) * g0 + __uint_as_float(b[4 * k + 3]) * g1;
-                if (single) d4[k] = v;
-                else {  // partial rows are (D + 2) floats: only 8-byte aligned
-                  float2* d2 = reinterpret_cast<float2*>(d4 + k);
-                  d2[0] = make_float2(v.x, v.y);
-                  d2[1] = make_float2(v.z, v.w);
-                }
-              }
+              for (int k = 0; k < 16; ++k)
+                dst[c * 32 + 2 * k + cpar] = __uint_as_float(a[k]) * g0 + __uint_as_float(b[k]) * g1;
             }
           }
-          if (!single && valid) {
-            dst[0] = M;
-            dst[1] = L;
+          if (!single && valid && cpar == 0) {
+            dst[-2] = M;
+            dst[-1] = L;
           }
         }
         tc::fence_before_sync();
@@ -475,16 +546,34 @@ bool make_kv_map(CUtensorMap* m, const void* base, long long rows, int D) {
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+int smem_optin() {
+  static int cached = -1;
+  if (cached < 0) {
+    int dev = 0, v = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+      v = 227 * 1024;
+    cached = v;
+  }
+  return cached;
+}
+
 template <int D>
 cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   using C = TcCfg<D>;
   static bool configured = false;
+  const int limit = smem_optin();
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)C::smem_bytes(kMaxBatch));
+    cudaError_t e =
+        cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
     if (e != cudaSuccess) return e;
     configured = true;
   }
+  // As many K/V stages as the shared memory holds, and an even number: K slot
+  // j % ns then only ever carries tiles of one parity, i.e. of one S issuer.
+  int ns = kMaxStages;
+  while (ns > 2 && C::smem_bytes(a.B, ns) > (size_t)limit) ns -= 2;
+  if (C::smem_bytes(a.B, ns) > (size_t)limit) return cudaErrorNotSupported;
   const long long rows = (long long)a.B * a.H * a.S_cap;
   CUtensorMap mk, mv;
   if (!make_kv_map(&mk, a.K, rows, D) || !make_kv_map(&mv, a.V, rows, D)) return cudaErrorNotSupported;
@@ -503,8 +592,9 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
   p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
+  p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B), st>>>(mk, mv, p);
+  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
   return cudaGetLastError();
 }
 
