@@ -134,6 +134,24 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ----------------------------------------------------------- multi-rank
+def max_over_ranks(x: float, device=None) -> float:
+    """The largest value of x over all ranks (x itself without a process group).
+    Timing takes the slowest rank, so a job's throughput is bounded by it."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank: float, world: int, seconds: float) -> float:
+    """Whole-job throughput of `world` replicas that each processed `units_per_rank`."""
+    return world * units_per_rank / seconds
+
+
 # ------------------------------------------------------- CPU oracle baseline
 def _oracle_pair(args):
     """Oracle for one (b, h) of the step: gamma cross-attention calls + the
@@ -319,17 +337,14 @@ def run_glide(args, rank, world, local_rank):
     per_kernel = {}
     for j, nm in enumerate(names):
         per_kernel.setdefault(nm, []).extend(ev[s][j][0].elapsed_time(ev[s][j][1]) for s in range(args.steps))
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, dev)
     if gb.glide_read_device_status(ws) != gb.GLIDE_OK or gb.glide_read_device_status(ws_acc) != gb.GLIDE_OK:
         raise RuntimeError("device status not OK after the timed region")
 
     cross_kv, verify_kv = kv_bytes(w)
     step_kv = w.gamma * cross_kv + verify_kv
-    value = world * step_kv * args.steps / (elapsed_ms * 1e-3) / 1e9
-    tree_tok = world * B * n * args.steps / (elapsed_ms * 1e-3)
+    value = job_throughput(step_kv * args.steps, world, elapsed_ms * 1e-3) / 1e9
+    tree_tok = job_throughput(B * n * args.steps, world, elapsed_ms * 1e-3)
 
     # ---- end to end: per-round inputs from pinned host memory, results back to host
     e2e_steps = max(3, min(args.steps, args.e2e_steps))
@@ -382,11 +397,8 @@ def run_glide(args, rank, world, local_rank):
     for _ in range(e2e_steps):
         e2e_step()
     e2e_s = time.perf_counter() - e0
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e_value = world * step_kv * e2e_steps / e2e_s / 1e9
+    e2e_s = max_over_ranks(e2e_s, dev)
+    e2e_value = job_throughput(step_kv * e2e_steps, world, e2e_s) / 1e9
 
     # ---- roofline of the dominant kernel
     peak, peak_src = measured_peaks()

@@ -186,6 +186,17 @@ glide_status glide_validate_tree(const int32_t* parent_idx_host, int32_t B, int3
                                  int32_t require_root0);
 
 /*
+ * Self-test of the failure path (no counterpart in the paper): launches one
+ * small kernel whose bounded waits on a barrier that nothing completes give up
+ * after limit_us microseconds (1 .. 2,000,000), record GLIDE_ERR_DEVICE_TIMEOUT
+ * in `workspace` (any attention or acceptance workspace) and release the
+ * kernel's other waiter, as every kernel of the library does when a wait runs
+ * out.  glide_read_device_status then returns that code and clears it.  The
+ * GPU neither faults nor hangs, and the context stays usable.
+ */
+glide_status glide_selftest_wait_timeout(void* workspace, uint32_t limit_us, glide_stream_t stream);
+
+/*
  * Waits for `stream`, then returns the status the kernels recorded in
  * `workspace` (GLIDE_OK or GLIDE_ERR_DEVICE_TIMEOUT) and clears it.  Works on
  * attention and acceptance workspaces alike.

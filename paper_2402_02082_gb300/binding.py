@@ -55,6 +55,7 @@ _SIG = {
     "glide_cross_attn_noalloc": (ctypes.c_int, [ctypes.POINTER(AttnDesc), _P, _P, _P, _P, ctypes.c_int32, _P, _P]),
     "glide_validate_tree": (ctypes.c_int, [_P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
     "glide_read_device_status": (ctypes.c_int, [_P, _P]),
+    "glide_selftest_wait_timeout": (ctypes.c_int, [_P, ctypes.c_uint32, _P]),
 }
 
 
@@ -209,3 +210,8 @@ def glide_validate_tree(parent_idx_host, require_root0: bool = True) -> int:
 
 def glide_read_device_status(workspace: torch.Tensor, stream=None) -> int:
     return int(lib().glide_read_device_status(workspace.data_ptr(), _stream(stream)))
+
+
+def glide_selftest_wait_timeout(workspace: torch.Tensor, limit_us: int, stream=None) -> int:
+    """Launch the bounded-wait self-test kernel (see include/glide.h); returns the launch status."""
+    return int(lib().glide_selftest_wait_timeout(workspace.data_ptr(), int(limit_us), _stream(stream)))
