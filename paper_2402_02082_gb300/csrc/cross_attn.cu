@@ -8,11 +8,13 @@
 // * persistent grid (one CTA per SM); the key ranges of all (b, h) are cut
 //   into 16-key tiles and dealt to CTAs in equal contiguous shares (split-KV
 //   with exact balance, ragged batches included);
-// * one producer thread streams K and V tiles with 1-D bulk copies (TMA) into
-//   shared-memory stages guarded by mbarriers; tile i goes to consumer warp
-//   i % NW, and every consumer warp owns a private ring of SW stages that it
-//   drains strictly in order (a warp never waits on a stage whose earlier
-//   phase is still pending, so the mbarrier parity cannot alias);
+// * four producer threads (one per producer warp; issuing a bulk copy keeps
+//   a thread busy for hundreds of cycles) stream K and V tiles with 1-D bulk
+//   copies (TMA) into shared-memory stages guarded by mbarriers; tile i goes
+//   to consumer warp i % NW, and every consumer warp owns a private ring of
+//   SW stages that it drains strictly in order (a warp never waits on a stage
+//   whose earlier phase is still pending, so the mbarrier parity cannot
+//   alias);
 // * each of the NW = 8 consumer warps (two per SM sub-partition, so one
 //   warp's shuffle and shared-memory latencies hide behind the other's work)
 //   takes whole tiles: lanes split the head dimension, a transpose-reduction
@@ -31,7 +33,8 @@ namespace {
 
 constexpr int kTK = 16;      // keys per tile
 constexpr int kNW = 8;       // consumer warps
-constexpr int kThreads = (kNW + 1) * 32;
+constexpr int kNP = 4;       // producer warps, each feeding kNW / kNP consumer rings
+constexpr int kThreads = (kNW + kNP) * 32;
 
 template <typename T, int D>
 struct CrossCfg {
@@ -107,8 +110,12 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
   const T* Kg = static_cast<const T*>(p.K);
   const T* Vg = static_cast<const T*>(p.V);
 
-  if (warp == kNW) {
-    // ------------------------------------------------------------ producer
+  if (warp >= kNW) {
+    // ----------------------------------------------------------- producers
+    // Issuing a bulk copy keeps the issuing thread busy for hundreds of cycles,
+    // so one thread cannot feed all the rings at HBM speed: producer pw feeds
+    // the rings of consumer warps kNW/kNP*pw .. kNW/kNP*(pw+1)-1.
+    const int pw = warp - kNW;
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       int i = 0;
@@ -117,6 +124,7 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
         const Segment s = locate(bt, P, p.B, g, g_end);
         const size_t slab = ((size_t)s.b * p.H + s.h) * p.S_cap;
         for (int t = s.t0; t < s.t1; ++t, ++i) {
+          if ((i % kNW) / (kNW / kNP) != pw) continue;  // another producer's ring
           const int r = i / kNW;  // use count of this warp's ring
           const int st = (i % kNW) * C::SW + r % C::SW;
           if (!mbar_wait(&empty[st], ((r / C::SW) & 1) ^ 1, abort_flag, p.status)) { ok = false; break; }
@@ -131,6 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
       }
       if (!ok) {  // let copies already issued land before the CTA exits
         for (int j = (i > NS ? i - NS : 0); j < i; ++j) {
+          if ((j % kNW) / (kNW / kNP) != pw) continue;
           const int r = j / kNW;
           mbar_drain(&full[(j % kNW) * C::SW + r % C::SW], (r / C::SW) & 1);
         }
