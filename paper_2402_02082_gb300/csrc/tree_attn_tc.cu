@@ -109,9 +109,12 @@ struct TcParams {
   float scale_log2;
 };
 
-// Lane 0 waits, the warp follows: every lane sees the same outcome, so the
-// warp-collective tcgen05 instructions that follow stay convergent.
+// Warp-uniform wait: every lane probes once and the warp votes; only if the
+// phase is not complete yet does lane 0 run the bounded wait and the warp
+// follow it.  Every lane sees the same outcome, so the warp-collective
+// tcgen05 instructions that follow stay convergent.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, unsigned* status) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
   int ok = 1;
   if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, status) ? 1 : 0;
   ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -361,14 +364,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
 
       float m_used = -CUDART_INF_F, l = 0.f;  // l: this thread's share of the row sum
+      // S of the next tile is loaded while this tile's exponentials run (within
+      // the segment only: the next segment's S needs a Q written after it ends)
+      uint32_t sr[16];
+      if (!dead) dead = !warp_wait(&bars[B_SFULL + i % kSBuf], (i / kSBuf) & 1, abort_flag, p.status);
+      if (!dead) {
+        tc::fence_after_sync();
+        tc::tmem_ld16x64b_x16(lane_addr + (i % kSBuf) * kTK + half * kHK, sr);
+      }
       for (int t = s.t0; t < s.t1; ++t, ++i) {
         const int j = i;
-        uint32_t sr[16];
-        if (!dead) dead = !warp_wait(&bars[B_SFULL + j % kSBuf], (j / kSBuf) & 1, abort_flag, p.status);
-        if (!dead) {
-          tc::fence_after_sync();
-          tc::tmem_ld16x64b_x16(lane_addr + (j % kSBuf) * kTK + half * kHK, sr);
-          tc::tmem_wait_ld();
+        tc::tmem_wait_ld();
+        uint32_t cur[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          asm volatile("" : "+r"(sr[k]));  // sr is only valid after the wait: keep reads below it
+          cur[k] = sr[k];
         }
         tc::fence_before_sync();
         __syncwarp();
@@ -379,13 +390,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         float sc[16];
         if (t * kTK + half * kHK + kHK <= plen) {
 #pragma unroll
-          for (int k = 0; k < 16; ++k) sc[k] = __uint_as_float(sr[k]) * sl2;
+          for (int k = 0; k < 16; ++k) sc[k] = __uint_as_float(cur[k]) * sl2;
         } else {
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
             const int key = key0 + 2 * k;
             const bool vis = key < plen || (key < len && ((anc >> ((key - plen) & 63)) & 1ull));
-            sc[k] = vis ? __uint_as_float(sr[k]) * sl2 : -CUDART_INF_F;
+            sc[k] = vis ? __uint_as_float(cur[k]) * sl2 : -CUDART_INF_F;
+          }
+        }
+        if (t + 1 < s.t1) {  // start loading S of the next tile
+          const int jn = j + 1;
+          if (!dead) dead = !warp_wait(&bars[B_SFULL + jn % kSBuf], (jn / kSBuf) & 1, abort_flag, p.status);
+          if (!dead) {
+            tc::fence_after_sync();
+            tc::tmem_ld16x64b_x16(lane_addr + (jn % kSBuf) * kTK + half * kHK, sr);
           }
         }
         float mx[4] = {sc[0], sc[1], sc[2], sc[3]};
