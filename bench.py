@@ -364,26 +364,52 @@ def run_glide(args, rank, world, local_rank):
     r_b = torch.empty(B, dtype=torch.int32).pin_memory()
     K16, V16 = K.view(torch.int16), V.view(torch.int16)
 
+    s_comp = torch.cuda.current_stream()
+    s_h2d = torch.cuda.Stream(device=dev)
+    s_d2h = torch.cuda.Stream(device=dev)
+
     def e2e_step():
-        kv_len.copy_(h_kv, non_blocking=True)
-        for b in range(B):
-            K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tk[b], non_blocking=True)
-            V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tv[b], non_blocking=True)
+        """One round through the public API with host buffers: inputs stream in
+        on a copy stream in the order they are needed, each call waits only for
+        its own inputs, and results stream back on a second copy stream."""
+        ev_in = []
+        with torch.cuda.stream(s_h2d):
+            kv_len.copy_(h_kv, non_blocking=True)
+            for b in range(B):
+                K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tk[b], non_blocking=True)
+                V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tv[b], non_blocking=True)
+            for i in range(w.gamma):
+                q_draft[i].view(torch.int16).copy_(h_qd[i], non_blocking=True)
+                ev_in.append(s_h2d.record_event())
+            q_tree.view(torch.int16).copy_(h_qt, non_blocking=True)
+            parent.copy_(h_par, non_blocking=True)
+            ev_tree = s_h2d.record_event()
+            draft.copy_(h_dr, non_blocking=True)
+            logits.copy_(h_lg, non_blocking=True)
+            ev_acc = s_h2d.record_event()
         for i in range(w.gamma):
-            q_draft[i].view(torch.int16).copy_(h_qd[i], non_blocking=True)
-            gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws)
-            r_c[i].copy_(out_c[i], non_blocking=True)
-        q_tree.view(torch.int16).copy_(h_qt, non_blocking=True)
-        parent.copy_(h_par, non_blocking=True)
-        gb.tree_verify_attn(q_tree, parent, K, V, kv_len, w.max_kv_len, out_t, ws, flags=flags)
-        r_t.copy_(out_t, non_blocking=True)
-        draft.copy_(h_dr, non_blocking=True)
-        logits.copy_(h_lg, non_blocking=True)
-        gb.tree_accept(draft, parent, logits, path, ln, bonus, ws_acc)
-        r_p.copy_(path, non_blocking=True)
-        r_l.copy_(ln, non_blocking=True)
-        r_b.copy_(bonus, non_blocking=True)
-        torch.cuda.synchronize()
+            s_comp.wait_event(ev_in[i])
+            gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws, stream=s_comp)
+            done = s_comp.record_event()
+            s_d2h.wait_event(done)
+            with torch.cuda.stream(s_d2h):
+                r_c[i].copy_(out_c[i], non_blocking=True)
+        s_comp.wait_event(ev_tree)
+        gb.tree_verify_attn(q_tree, parent, K, V, kv_len, w.max_kv_len, out_t, ws, flags=flags, stream=s_comp)
+        done = s_comp.record_event()
+        s_d2h.wait_event(done)
+        with torch.cuda.stream(s_d2h):
+            r_t.copy_(out_t, non_blocking=True)
+        s_comp.wait_event(ev_acc)
+        gb.tree_accept(draft, parent, logits, path, ln, bonus, ws_acc, stream=s_comp)
+        done = s_comp.record_event()
+        s_d2h.wait_event(done)
+        with torch.cuda.stream(s_d2h):
+            r_p.copy_(path, non_blocking=True)
+            r_l.copy_(ln, non_blocking=True)
+            r_b.copy_(bonus, non_blocking=True)
+        s_d2h.synchronize()
+        s_comp.synchronize()
 
     h2d = (sum(t.numel() * t.element_size() for t in h_qd) + h_qt.numel() * h_qt.element_size() +
            h_par.numel() * 4 + h_kv.numel() * 4 + h_dr.numel() * 4 + h_lg.numel() * 4 +
