@@ -15,6 +15,11 @@ It is a plain, slow, fp64 restatement of what the path computes:
 * ``accept.tree_accept``         -- greedy acceptance (speculative decoding,
   Section 2) on a token tree: the deepest node whose root path the target's
   argmax reproduces, plus the free bonus token.
+* ``cape.cape_expand``           -- CaPE's confidence-aware proposal expansion
+  (Section 3.2; the fixed-size variant of Section 4): proposal tokens, S(p_i)
+  sized expansion sets, and the linearized token tree.
+* ``kvcache.kv_compact``         -- the cache update after verification
+  (Section 3.1): the accepted path's entries become contiguous rows.
 
 Every function here is pinned by tests in ``tests/test_oracle.py`` against
 closed forms, library routines, brute force and invariants; none is marked
@@ -23,6 +28,8 @@ closed forms, library routines, brute force and invariants; none is marked
 from .attention import (ancestors_or_self, cape_mask, cross_attn, tree_allowed_mask,
                         tree_verify_attn, widen)
 from .accept import row_argmax, tree_accept
+from .cape import cape_expand, expansion_size
+from .kvcache import kv_compact
 
 __all__ = ["ancestors_or_self", "cape_mask", "cross_attn", "tree_allowed_mask",
-           "tree_verify_attn", "widen", "row_argmax", "tree_accept"]
+           "tree_verify_attn", "widen", "row_argmax", "tree_accept", "cape_expand", "expansion_size", "kv_compact"]

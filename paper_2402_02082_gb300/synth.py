@@ -149,6 +149,36 @@ def planted_logits(seed: int, parent: np.ndarray, tokens: np.ndarray, vocab: int
     return lg
 
 
+def draft_probs(seed: int, B: int, gamma: int, vocab: int, quantum: float = 0.0) -> np.ndarray:
+    """fp32 draft distributions [B, gamma, vocab] for proposal expansion.
+
+    Each row's largest entry (the confidence) is drawn uniformly from
+    [0.05, 0.98], so the four confidence bands of CaPE's size rule are all
+    visited; the remaining mass is spread over the other tokens with a
+    heavy-tailed (Gamma(0.3)) profile, as an LLM's next-token distribution
+    has a few runners-up and a long flat tail.  With quantum > 0 every entry
+    is rounded to a multiple of it, which creates many exact ties (and zeros).
+    """
+    g = _rng(seed, 31)
+    out = np.empty((B, gamma, vocab), dtype=np.float32)
+    for b in range(B):
+        for i in range(gamma):
+            conf = g.uniform(0.05, 0.98)
+            tail = g.gamma(0.3, size=vocab - 1)
+            tail *= (1.0 - conf) / tail.sum()
+            tail = np.minimum(tail, conf)
+            row = np.insert(tail, int(g.integers(vocab)), conf)
+            if quantum > 0:
+                row = np.round(row / quantum) * quantum
+            out[b, i] = row
+    return out
+
+
+def root_tokens(seed: int, B: int, vocab: int) -> np.ndarray:
+    """x_t of each sequence (the token the next tree hangs from)."""
+    return _rng(seed, 32).integers(vocab, size=B).astype(np.int32)
+
+
 # --------------------------------------------------------------------------
 # workloads
 # --------------------------------------------------------------------------

@@ -346,3 +346,242 @@ def check_argmax_ties(row_argmax):
     lg = np.array([[1.0, 3.0, 3.0, 2.0], [5.0, 5.0, 5.0, 5.0], [-1.0, -2.0, -1.0, -3.0],
                    [0.0, -0.0, 0.0, -1.0]], dtype=np.float32)
     assert list(row_argmax(lg)) == [1, 0, 0, 0]
+
+
+# ----------------------------------------------------------- CaPE expansion
+def read_cape_expand_golden():
+    examples, sizes, cur, case = [], [], None, None
+    for ln in open(os.path.join(GOLDEN, "cape_expand_examples.txt")):
+        ln = ln.strip()
+        if not ln or ln.startswith("#"):
+            continue
+        key, *vals = ln.split()
+        if key == "example":
+            cur = {"name": vals[0], "prob": [], "cases": []}
+            examples.append(cur)
+        elif key == "root":
+            cur["root"] = int(vals[0])
+        elif key == "prob":
+            cur["prob"].append([float(v) for v in vals])
+        elif key == "case":
+            case = {"max_tokens": int(vals[0]), "fixed": None if vals[1] == "-" else int(vals[1])}
+            cur["cases"].append(case)
+        elif key == "size":
+            bits = np.array([int(vals[0], 16)], dtype=np.uint32)
+            sizes.append((float(bits.view(np.float32)[0]), int(vals[1])))
+        else:
+            case[key] = [int(v) for v in vals]
+    return examples, sizes
+
+
+def check_cape_expand_golden(cape_expand, expansion_size):
+    """The hand-worked expansions (basic, caps, fixed size 4, tie + clamp) and
+    S(p) at the binary32 neighbours of its thresholds."""
+    examples, sizes = read_cape_expand_golden()
+    for p, k in sizes:
+        assert expansion_size(np.float32(p)) == k, f"S({p!r})"
+    for ex in examples:
+        probs = np.array([ex["prob"]], dtype=np.float32)
+        gamma = probs.shape[1]
+        for case in ex["cases"]:
+            tok, par, nn, conf, ku = cape_expand(probs, np.array([ex["root"]]), case["max_tokens"],
+                                                 case["fixed"])
+            m = len(case["tokens"])
+            tag = f"{ex['name']} cap {case['max_tokens']} fixed {case['fixed']}"
+            assert int(nn[0]) == m, tag
+            assert list(tok[0, :m]) == case["tokens"], tag
+            assert list(par[0, :m]) == case["parent"], tag
+            assert list(ku[0]) == case["k"], tag
+            assert all(tok[0, m:] == -1) and all(par[0, m:] == 0), tag + " padding"
+            assert np.array_equal(conf[0], probs[0].max(axis=-1)), tag + " conf"
+            assert tok.shape[1] == 1 + case["max_tokens"], tag
+            assert gamma <= case["max_tokens"]
+
+
+def _outranks(p, a, b):
+    """Token a ranks before token b in distribution p (ties: lower id)."""
+    pa, pb = float(p[a]) + 0.0, float(p[b]) + 0.0
+    return pa > pb or (pa == pb and a < b)
+
+
+def check_cape_expand_brute_force(cape_expand, expansion_size):
+    """Tiny vocabularies with many ties: x_{t+i} outranks every other token and
+    X_i is the one subset of its size whose members all outrank every
+    non-member, found by enumerating all subsets."""
+    g = _rng(20)
+    levels = np.array([0.0, 0.05, 0.1, 0.2, 0.35, 0.65, 0.9], dtype=np.float32)
+    for trial in range(200):
+        V = int(g.integers(2, 9))
+        gamma = int(g.integers(1, 4))
+        probs = levels[g.integers(len(levels), size=(1, gamma, V))]
+        tok, par, nn, conf, ku = cape_expand(probs, np.array([0]), 63)
+        node = gamma + 1
+        for i in range(1, gamma + 1):
+            p = probs[0, i - 1]
+            x = int(tok[0, i])
+            assert all(_outranks(p, x, u) for u in range(V) if u != x), f"trial {trial} x"
+            k = int(ku[0, i - 1])
+            assert k == min(expansion_size(p[x]), V - 1), f"trial {trial} K"
+            X = [int(t) for t in tok[0, node:node + k]]
+            assert all(int(q) == i - 1 for q in par[0, node:node + k]), f"trial {trial} parent"
+            node += k
+            others = [u for u in range(V) if u != x]
+            winners = [set(T) for T in itertools.combinations(others, k)
+                       if all(_outranks(p, a, b) for a in T for b in others if b not in T)]
+            assert len(winners) == 1 and set(X) == winners[0], f"trial {trial} set"
+            assert all(_outranks(p, X[r], X[r + 1]) for r in range(k - 1)), f"trial {trial} order"
+        assert int(nn[0]) == node
+
+
+def _planted_rows(g, sizes, V):
+    """One distribution per position whose maximum is a value with a known
+    S(p) from Section 3.2's table; the rest of the mass is spread below it."""
+    p_of_size = {1: 0.9, 3: 0.7, 5: 0.5, 7: 0.2}
+    rows = []
+    for k in sizes:
+        pmax = p_of_size[k]
+        rest = g.random(V - 1) + 0.5
+        rest *= (1.0 - pmax) / rest.sum()
+        row = np.insert(rest, int(g.integers(V)), pmax)
+        rows.append(row)
+    return np.array([rows], dtype=np.float32)
+
+
+def check_cape_expand_mask(cape_expand, cape_mask, tree_allowed_mask):
+    """The tree built from CaPE's sets, under the ancestor-or-self rule, gives
+    exactly the CaPE mask equation of Section 3.2 for the linearized proposal
+    (pos() from the set sizes the planted confidences dictate)."""
+    g = _rng(21)
+    for _ in range(60):
+        gamma = int(g.integers(1, 6))
+        sizes = [int(k) for k in g.choice([1, 3, 5, 7], size=gamma)]
+        probs = _planted_rows(g, sizes, 64)
+        tok, par, nn, conf, ku = cape_expand(probs, np.array([5]), 63)
+        assert list(ku[0]) == sizes
+        n = int(nn[0])
+        assert n == 1 + gamma + sum(sizes)
+        pos = [0] + list(range(1, gamma + 1)) + [j for j, k in enumerate(sizes, start=1) for _ in range(k)]
+        allowed = tree_allowed_mask(par[0, :n], 0)
+        assert np.array_equal(allowed[1:, 1:], cape_mask(gamma, pos)), "CaPE tree mask"
+        # siblings are distinct tokens, so greedy acceptance has one answer
+        for p in range(n):
+            kids = [int(tok[0, c]) for c in range(1, n) if par[0, c] == p]
+            assert len(kids) == len(set(kids)), "duplicate siblings"
+
+
+def check_cape_expand_cap(cape_expand):
+    """Under a binding cap every dropped expansion token ranks after every kept
+    one (probability, then position, then rank), each kept set is a prefix of
+    its uncapped set, and the fixed size 0 gives the plain proposal chain."""
+    g = _rng(22)
+    for trial in range(100):
+        gamma = int(g.integers(1, 6))
+        V = int(g.integers(10, 60))
+        probs = g.dirichlet(np.full(V, 0.3), size=(1, gamma)).astype(np.float32)
+        probs[0, :, :3] = np.round(probs[0, :, :3], 1)           # some cross-position ties
+        full = cape_expand(probs, np.array([1]), 63)
+        cap = int(g.integers(gamma, gamma + int(full[4].sum()) + 1))
+        part = cape_expand(probs, np.array([1]), cap)
+
+        def entries(res):
+            tok, par, nn, conf, ku = res
+            out, node = [], gamma + 1
+            for i in range(1, gamma + 1):
+                for r in range(int(ku[0, i - 1])):
+                    t = int(tok[0, node])
+                    out.append((float(probs[0, i - 1, t]) + 0.0, i, r, t))
+                    node += 1
+            return out
+
+        e_full, e_part = entries(full), entries(part)
+        kept = set(e_part)
+        assert kept <= set(e_full), f"trial {trial}"
+        assert len(e_part) == min(len(e_full), cap - gamma), f"trial {trial}"
+        for i in range(1, gamma + 1):
+            mine = [e for e in e_full if e[1] == i]
+            km = [e for e in e_part if e[1] == i]
+            assert km == mine[:len(km)], f"trial {trial} prefix"
+        for d in set(e_full) - kept:
+            for k in kept:
+                assert (k[0] > d[0]) or (k[0] == d[0] and (k[1], k[2]) < (d[1], d[2])), f"trial {trial} order"
+        assert np.array_equal(full[0][0, :gamma + 1], part[0][0, :gamma + 1])
+        chain = cape_expand(probs, np.array([1]), gamma, fixed_k=0)
+        assert int(chain[2][0]) == gamma + 1 and list(chain[1][0]) == [-1] + list(range(gamma))
+
+
+# --------------------------------------------------------- KV-cache update
+def read_kv_golden():
+    seqs, cur = [], None
+    for ln in open(os.path.join(GOLDEN, "kv_compact_example.txt")):
+        ln = ln.strip()
+        if not ln or ln.startswith("#"):
+            continue
+        key, *vals = ln.split()
+        if key == "seq":
+            cur = {}
+            seqs.append(cur)
+        else:
+            cur[key] = [int(v) for v in vals]
+    return seqs
+
+
+def check_kv_compact_golden(kv_compact):
+    seqs = read_kv_golden()
+    B, S = len(seqs), len(seqs[0]["rows"])
+    K = np.array([[s["rows"]] for s in seqs], dtype=np.float32)[..., None]    # [B, 1, S, 1]
+    V = -K
+    n = max(len(s["path"]) for s in seqs)
+    path = np.full((B, n), -1, dtype=np.int32)
+    for b, s in enumerate(seqs):
+        path[b, :len(s["path"])] = s["path"]
+    K2, V2, nl = kv_compact(K, V, [s["kv_len"][0] for s in seqs], path, [s["len"][0] for s in seqs])
+    for b, s in enumerate(seqs):
+        assert list(K2[b, 0, :, 0].astype(int)) == s["want"], f"seq {b} K"
+        assert list((-V2[b, 0, :, 0]).astype(int)) == s["want"], f"seq {b} V"
+        assert int(nl[b]) == s["new_len"][0], f"seq {b} length"
+    assert S == K2.shape[2]
+
+
+def check_kv_compact_attention(kv_compact, tree_verify_attn, cross_attn):
+    """The kept cache is exactly what the accepted node attended to during
+    verification: plain attention of that node's query over the compacted
+    cache reproduces its tree-attention output (up to fp64 rounding)."""
+    g = _rng(23)
+    for _ in range(20):
+        B, H, D = 2, 2, 8
+        n = int(g.integers(1, 10))
+        L = [int(g.integers(0, 12)) for _ in range(B)]
+        S = max(L) + n + 2
+        K = g.standard_normal((B, H, S, D)).astype(np.float32)
+        V = g.standard_normal((B, H, S, D)).astype(np.float32)
+        parent = np.stack([random_small_tree(g, n) for _ in range(B)])
+        q = g.standard_normal((B, n, H, D)).astype(np.float32)
+        ref = tree_verify_attn(q, parent, K, V, L)
+        path = np.full((B, n), -1, dtype=np.int32)
+        length, node = [], []
+        for b in range(B):
+            c = int(g.integers(n))
+            chain = [c]
+            while chain[-1] != 0:
+                chain.append(int(parent[b, chain[-1]]))
+            chain = chain[::-1]
+            path[b, :len(chain)] = chain
+            length.append(len(chain) - 1)
+            node.append(c)
+        K2, V2, nl = kv_compact(K, V, L, path, length)
+        qd = np.stack([q[b, node[b]] for b in range(B)])[:, None]
+        got = cross_attn(qd, K2, V2, nl)
+        for b in range(B):
+            assert np.allclose(got[b, 0], ref[b, node[b]], rtol=1e-12, atol=1e-12), "kept cache"
+
+
+def check_kv_compact_chain_identity(kv_compact):
+    """Accepting a chain prefix (path[k] = k) moves nothing: the buffers are
+    returned unchanged and only the length grows."""
+    g = _rng(24)
+    K = g.standard_normal((3, 2, 4, 20, 8)).astype(np.float32)     # [layers, B, H, S, D]
+    V = g.standard_normal((3, 2, 4, 20, 8)).astype(np.float32)
+    path = np.array([[0, 1, 2, -1, -1, -1], [0, 1, 2, 3, 4, 5]], dtype=np.int32)
+    K2, V2, nl = kv_compact(K, V, [3, 10], path, [2, 5])
+    assert np.array_equal(K2, K) and np.array_equal(V2, V)
+    assert list(nl) == [6, 16]

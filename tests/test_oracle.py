@@ -206,3 +206,121 @@ def test_mutant_accept_ignores_ancestors():
             bo[b] = a[b][best]
         return path, ln, bo
     _expect_some_fail([lambda: pins.check_accept_brute_force(bad), lambda: pins.check_accept_golden(bad)])
+
+
+# ----------------------------------------------------------- CaPE expansion
+from oracle import cape as ocape
+from oracle import kvcache as okv
+
+
+def test_cape_expand_golden():
+    pins.check_cape_expand_golden(ocape.cape_expand, ocape.expansion_size)
+
+
+def test_cape_expand_brute_force():
+    pins.check_cape_expand_brute_force(ocape.cape_expand, ocape.expansion_size)
+
+
+def test_cape_expand_mask():
+    pins.check_cape_expand_mask(ocape.cape_expand, oracle.cape_mask, oracle.tree_allowed_mask)
+
+
+def test_cape_expand_cap():
+    pins.check_cape_expand_cap(ocape.cape_expand)
+
+
+def _cape_pins():
+    return [lambda: pins.check_cape_expand_golden(ocape.cape_expand, ocape.expansion_size),
+            lambda: pins.check_cape_expand_brute_force(ocape.cape_expand, ocape.expansion_size),
+            lambda: pins.check_cape_expand_mask(ocape.cape_expand, oracle.cape_mask,
+                                                oracle.tree_allowed_mask),
+            lambda: pins.check_cape_expand_cap(ocape.cape_expand)]
+
+
+def test_mutant_s_thresholds_in_fp32(monkeypatch):
+    # comparing with the thresholds rounded to binary32 (p <= 0.3f) puts
+    # 0.3f = 0.3000000119... in the first bucket
+    def fp32_thresholds(p):
+        x = np.float32(p)
+        for upper, k in ocape._S_TABLE:
+            if x <= np.float32(float(upper)):
+                return k
+        return ocape._S_LAST
+    monkeypatch.setattr(ocape, "expansion_size", fp32_thresholds)
+    _expect_some_fail(_cape_pins())
+
+
+def test_mutant_set_keeps_proposal_token(monkeypatch):
+    monkeypatch.setattr(ocape, "expansion_set", lambda order, k: order[0:k])
+    _expect_some_fail(_cape_pins())
+
+
+def test_mutant_ties_to_higher_id(monkeypatch):
+    def ranked(row):
+        vals = [float(v) + 0.0 for v in row]
+        return sorted(range(len(vals)), key=lambda t: (-vals[t], -t))
+    monkeypatch.setattr(ocape, "ranked_tokens", ranked)
+    _expect_some_fail(_cape_pins())
+
+
+def test_mutant_cap_cuts_linearized_tail(monkeypatch):
+    monkeypatch.setattr(ocape, "keep_after_cap",
+                        lambda cands, room: sorted(cands, key=lambda c: (c[1], c[2]))[:room])
+    _expect_some_fail(_cape_pins())
+
+
+def test_mutant_expansion_under_proposal_token(monkeypatch):
+    real = ocape.cape_expand
+
+    def bad(probs, root, max_tokens=32, fixed_k=None):
+        tok, par, nn, conf, ku = real(probs, root, max_tokens, fixed_k)
+        gamma = probs.shape[1]
+        for b in range(len(nn)):
+            par[b, gamma + 1:nn[b]] += 1          # child of x_{t+i} instead of its sibling
+        return tok, par, nn, conf, ku
+    monkeypatch.setattr(ocape, "cape_expand", bad)
+    _expect_some_fail(_cape_pins())
+
+
+# --------------------------------------------------------- KV-cache update
+def test_kv_compact_golden():
+    pins.check_kv_compact_golden(okv.kv_compact)
+
+
+def test_kv_compact_attention():
+    pins.check_kv_compact_attention(okv.kv_compact, oracle.tree_verify_attn, oracle.cross_attn)
+
+
+def test_kv_compact_chain_identity():
+    pins.check_kv_compact_chain_identity(okv.kv_compact)
+
+
+def _kv_pins(fn):
+    return [lambda: pins.check_kv_compact_golden(fn),
+            lambda: pins.check_kv_compact_attention(fn, oracle.tree_verify_attn, oracle.cross_attn),
+            lambda: pins.check_kv_compact_chain_identity(fn)]
+
+
+def test_mutant_kv_length_without_root():
+    def bad(K, V, kv_len, path, length):
+        K2, V2, nl = okv.kv_compact(K, V, kv_len, path, length)
+        return K2, V2, nl - 1
+    _expect_some_fail(_kv_pins(bad))
+
+
+def test_mutant_kv_skips_root_entry():
+    def bad(K, V, kv_len, path, length):
+        shifted = np.concatenate([path[:, 1:], np.full((path.shape[0], 1), -1, path.dtype)], axis=1)
+        shifted[shifted < 0] = 0
+        return okv.kv_compact(K, V, kv_len, shifted, length)
+    _expect_some_fail(_kv_pins(bad))
+
+
+def test_mutant_kv_reversed_path():
+    def bad(K, V, kv_len, path, length):
+        rev = path.copy()
+        for b in range(path.shape[0]):
+            m = int(length[b]) + 1
+            rev[b, :m] = path[b, :m][::-1]
+        return okv.kv_compact(K, V, kv_len, rev, length)
+    _expect_some_fail(_kv_pins(bad))
