@@ -246,6 +246,85 @@ def workload_config(w):
 
 
 # -------------------------------------------------------------------- main
+CAPE_MAX_TOKENS = 32   # the cap on verified tokens of the paper's CaPE runs (Section 4)
+
+
+def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
+    """CaPE expansion of this workload's gamma draft distributions over the
+    Vicuna vocabulary, and the cache update of one accepted path per tree,
+    each launched `args.next_iters` times with L2 flushed before
+    every launch; CUDA-event time of the launch alone."""
+    import torch
+    iters = max(3, args.next_iters)
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)   # > 129 MB L2
+
+    def timed(fn):
+        times = []
+        for _ in range(iters + 2):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            times.append((a, b))
+        torch.cuda.synchronize()
+        ms = [a.elapsed_time(b) for a, b in times[2:]]
+        return sum(ms) / len(ms)
+
+    B = w.B
+    probs = torch.from_numpy(synth.draft_probs(w.seed + 17, B, w.gamma, w.vocab)).to(dev)
+    roots = torch.from_numpy(synth.root_tokens(w.seed + 17, B, w.vocab)).to(dev)
+    n_out = 1 + CAPE_MAX_TOKENS
+    tok = torch.empty(B, n_out, dtype=torch.int32, device=dev)
+    par = torch.empty(B, n_out, dtype=torch.int32, device=dev)
+    nn = torch.empty(B, dtype=torch.int32, device=dev)
+    conf = torch.empty(B, w.gamma, device=dev)
+    ws_c = torch.zeros(gb.glide_cape_workspace_bytes(B, w.gamma, w.vocab), dtype=torch.uint8, device=dev)
+    cape_ms = timed(lambda: gb.cape_expand(probs, roots, CAPE_MAX_TOKENS, tok, par, nn, ws_c, conf=conf))
+    cape_bytes = probs.numel() * 4 + B * 4 + 2 * B * n_out * 4 + B * 4 + B * w.gamma * 4
+    nodes = nn.cpu().tolist()
+
+    # Accepted paths for the cache update: the step's own acceptance on random
+    # logits accepts almost nothing, so take, in each tree, the root path to the
+    # highest-numbered node of depth min(4, tree depth): an accepted length
+    # like the 3-4 tokens per round of the paper's CaPE runs, with every
+    # accepted entry moving.
+    par_h = case["parent_idx"]
+    n = par_h.shape[1]
+    p_h = np.full((B, n), -1, dtype=np.int32)
+    l_h = np.zeros(B, dtype=np.int32)
+    for b in range(B):
+        depth = synth.tree_depths(par_h[b])
+        d = min(4, int(depth.max()))
+        c = max(i for i in range(n) if depth[i] == d)
+        chain = [c]
+        while chain[-1] != 0:
+            chain.append(int(par_h[b, chain[-1]]))
+        p_h[b, :len(chain)] = chain[::-1]
+        l_h[b] = len(chain) - 1
+    path_c = torch.from_numpy(p_h).to(dev)
+    len_c = torch.from_numpy(l_h).to(dev)
+    new_len = torch.empty(B, dtype=torch.int32, device=dev)
+    comp_ms = timed(lambda: gb.glide_kv_compact(K, V, kv_len, path_c, len_c, new_len))
+    e = 2 if w.dtype == "bf16" else 4
+    moved = sum(1 for b in range(B) for k in range(1, int(l_h[b]) + 1) if int(p_h[b, k]) != k)
+    comp_bytes = moved * w.H * w.D * e * 2 * 2 + B * (4 * 3 + 4 * (int(l_h.max()) + 1))
+    del flush
+    return {
+        "cape_expand": {"avg_us": 1e3 * cape_ms, "algo_bytes_per_launch": cape_bytes,
+                        "achieved_gbs": cape_bytes / (cape_ms * 1e-3) / 1e9,
+                        "frac_of_peak": cape_bytes / (cape_ms * 1e-3) / 1e9 / peak,
+                        "shape": f"B={B} gamma={w.gamma} V={w.vocab} fp32, cap {CAPE_MAX_TOKENS}",
+                        "tree_nodes": nodes},
+        "glide_kv_compact": {"avg_us": 1e3 * comp_ms, "algo_bytes_per_launch": comp_bytes,
+                             "achieved_gbs": comp_bytes / (comp_ms * 1e-3) / 1e9,
+                             "frac_of_peak": comp_bytes / (comp_ms * 1e-3) / 1e9 / peak,
+                             "moved_rows": moved, "accepted_len": [int(x) for x in l_h],
+                             "shape": f"one layer, B={B} H={w.H} D={w.D} {w.dtype}"},
+        "iters": iters, "l2": "flushed before every launch",
+    }
+
+
 def run_glide(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -426,8 +505,13 @@ def run_glide(args, rank, world, local_rank):
     e2e_s = max_over_ranks(e2e_s, dev)
     e2e_value = job_throughput(step_kv * e2e_steps, world, e2e_s) / 1e9
 
-    # ---- roofline of the dominant kernel
+    # ---- the calls around the round: CaPE expansion (before verification) and
+    # the cache update (after acceptance), each timed alone with L2 flushed
     peak, peak_src = measured_peaks()
+    next_rows = time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak)
+
+    # ---- roofline of the dominant kernel
+
     ab = algo_bytes(w)
     kernels = {}
     for nm, times in per_kernel.items():
@@ -444,7 +528,7 @@ def run_glide(args, rank, world, local_rank):
     cpu_baseline = None
     if cpu is not None:
         pool, cores = cpu
-        pairs = pick_pairs(w, args.cpu_pairs, 1234)
+        pairs = pick_pairs(w, args.cpu_pairs or w.B * w.H, 1234)
         gbs, dt = time_oracle(w, case, pairs, pool, cores)
         pool.close()
         cpu_baseline = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
@@ -460,7 +544,7 @@ def run_glide(args, rank, world, local_rank):
                 "frac_of_nominal_8tbs": value / world / NOMINAL_HBM_GBS,
                 "frac_of_measured_hbm": value / world / peak,
                 "tree_tokens_per_s_per_layer": tree_tok,
-                "roofline": roof, "kernels": kernels, "cpu_baseline": cpu_baseline,
+                "roofline": roof, "kernels": kernels, "next_rows": next_rows, "cpu_baseline": cpu_baseline,
                 "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                         "steps": e2e_steps},
                 "gpu_launches": len(step_fns) * args.steps, "clocks": clk}
@@ -480,7 +564,10 @@ def main():
     ap.add_argument("--impl", choices=["glide", "reference"], default="glide")
     ap.add_argument("--workload", default="vicuna33b-long-b4", choices=[w.name for w in synth.workloads()])
     ap.add_argument("--e2e-steps", type=int, default=50)
-    ap.add_argument("--cpu-pairs", type=int, default=64)
+    ap.add_argument("--next-iters", type=int, default=50,
+                    help="launches of each of cape_expand and glide_kv_compact timed after the step")
+    ap.add_argument("--cpu-pairs", type=int, default=0,
+                    help="(b, h) slabs in the CPU-baseline sample; 0 = every slab of one step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--force-fma", action="store_true")
     ap.add_argument("--batch", type=int, default=0,

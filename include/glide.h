@@ -17,6 +17,15 @@
  *                      deepest node whose whole root path the target's argmax
  *                      reproduces, and the free bonus token.
  *
+ * Two more calls close the round around them:
+ *
+ *   cape_expand        CaPE's confidence-aware proposal expansion (Section
+ *                      3.2): from the draft's distributions, the proposal
+ *                      tokens, the expansion sets and the linearized tree that
+ *                      tree_verify_attn and tree_accept take.
+ *   glide_kv_compact   the cache update after acceptance (Section 3.1): the
+ *                      accepted path's keys/values become contiguous rows.
+ *
  * Conventions shared by all calls
  * -------------------------------
  * - Every tensor pointer is a DEVICE pointer owned by the caller; the library
@@ -152,6 +161,73 @@ glide_status tree_accept(const int32_t* draft_tokens, const int32_t* parent_idx,
                          const float* target_logits, int32_t B, int32_t n, int32_t V,
                          int32_t* path, int32_t* len, int32_t* bonus,
                          void* workspace, size_t workspace_bytes, glide_stream_t stream);
+
+/* Bytes of workspace that cape_expand needs for B proposals of gamma
+ * positions over a vocabulary of V; 0 if the sizes are out of range. */
+size_t glide_cape_workspace_bytes(int32_t B, int32_t gamma, int32_t V);
+
+/*
+ * CaPE confidence-aware proposal expansion (Section 3.2; the fixed-size
+ * variant of Section 4's ablation with fixed_k >= 0):
+ *   for each sequence b and position i = 1..gamma, from the draft's
+ *   distribution probs[b,i-1,:]:
+ *     x_{t+i} = the most probable token, p_i = its probability (conf[b,i-1]);
+ *     K_i = S(p_i) = 7, 5, 3, 1 for p_i in (0,0.3], (0.3,0.6], (0.6,0.8], (0.8,1]
+ *           (exact comparison of the fp32 value with the decimal thresholds;
+ *           p_i <= 0 gives 7, p_i > 1 gives 1), or fixed_k; at most V-1;
+ *     X_i  = the K_i most probable tokens other than x_{t+i}.
+ *   Ranking: higher probability first, then the lower token id; -0 == +0.
+ *   Cap: the proposal and the sets hold at most max_tokens tokens (x_t not
+ *   counted); when the sets overflow, the expansion tokens of lowest
+ *   probability are dropped first (equal probabilities: the later position,
+ *   then the later rank), so every kept set is still the top of its position.
+ * Output: the linearized tree of n_out = 1 + max_tokens node slots per sequence,
+ *   draft_tokens [B, n_out], parent_idx [B, n_out] int32:
+ *     node 0          = root_token[b] (x_t), parent -1;
+ *     node i, 1..gamma = x_{t+i}, parent i-1;
+ *     then each position's kept set in position order, best first, every
+ *     token with parent i-1 (a sibling of x_{t+i});
+ *     unused slots n_nodes[b] .. n_out-1: token -1, parent 0 (a leaf that
+ *     acceptance never takes, since no argmax equals -1).
+ *   n_nodes [B] int32 = 1 + gamma + kept expansion tokens.
+ *   conf [B, gamma] fp32 = p_i (a zero is reported as +0), or NULL.
+ *   The ancestor-or-self mask of this tree is the CaPE mask of Section 3.2, so
+ *   the arrays go to tree_verify_attn and tree_accept as they are (n = n_out).
+ * probs [B, gamma, V] fp32 on the device, finite, 16-byte aligned;
+ * root_token [B] int32 on the device.  1 <= gamma <= max_tokens <= 63;
+ * fixed_k = -1 for S(p), or 0 .. 7 (larger: GLIDE_ERR_UNSUPPORTED).
+ */
+glide_status cape_expand(const float* probs, const int32_t* root_token, int32_t B, int32_t gamma,
+                         int32_t V, int32_t max_tokens, int32_t fixed_k, int32_t* draft_tokens,
+                         int32_t* parent_idx, int32_t* n_nodes, float* conf, void* workspace,
+                         size_t workspace_bytes, glide_stream_t stream);
+
+/*
+ * Cache update after acceptance (Section 3.1: the target keeps the cache
+ * entries of the accepted tokens and discards the rejected ones), in place,
+ * for n_layers layers at once:
+ *   for every layer, sequence b and head h, and k = 0 .. len[b]:
+ *     K[b,h,kv_len[b]+k,:] <- K[b,h,kv_len[b]+path[b,k],:]   (same for V)
+ *   new_kv_len[b] = kv_len[b] + len[b] + 1.
+ * This keeps x_t (node 0) and the accepted proposal tokens, in path order;
+ * the new bonus token has no entry yet (it is node 0 of the next tree).
+ * Every other row keeps its contents.
+ * desc: B, H, D, S_cap and dtype of one layer's cache (scale, flags and
+ * max_ctas are ignored).  K_cache/V_cache: layer 0 of [n_layers][B,H,S_cap,D];
+ * layer l starts layer_stride ELEMENTS after layer l-1 (layer_stride >=
+ * B*H*S_cap*D and a multiple of 16 bytes when n_layers > 1; ignored when 1).
+ * kv_len [B] (clamped to [0, S_cap-n]), path [B,n] (root-first node indices
+ * as tree_accept writes them, clamped to [0, n)), len [B] (clamped to
+ * [0, n-1]) are int32 on the device; 1 <= n <= 64, n <= S_cap.
+ * new_kv_len [B] int32 on the device and not the kv_len buffer (the kernel
+ * reads kv_len while it writes new_kv_len).  No workspace.
+ * Correct for every path that tree_accept produces (node indices along a root
+ * path are increasing); other paths stay in bounds but give unspecified rows.
+ */
+glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int64_t layer_stride,
+                              void* K_cache, void* V_cache, const int32_t* kv_len, int32_t n,
+                              const int32_t* path, const int32_t* len, int32_t* new_kv_len,
+                              glide_stream_t stream);
 
 /*
  * glide_cross_attn for callers that cannot allocate device memory when they

@@ -15,7 +15,7 @@ fixed size (4); ``fixed_k`` gives that variant.
 
 Readings where the paper is silent (each fixes an integer result exactly):
 * ranking is by probability, highest first, ties to the lower token id;
-  -0.0 and +0.0 are equal;
+  -0.0 and +0.0 are the same probability (a zero confidence is reported as +0);
 * the comparison with the decimal thresholds is exact: the fp32 value of p_i
   against the real number 0.3, 0.6 or 0.8 (none of which is a binary32 value,
   so whether an interval end is open or closed never matters for fp32 input);
@@ -104,7 +104,7 @@ def cape_expand(probs: np.ndarray, root_token: np.ndarray, max_tokens: int = 32,
             x = order[0]
             p = row[x]
             spine.append(x)
-            conf[b, i - 1] = p
+            conf[b, i - 1] = float(p) + 0.0           # a zero confidence is +0
             k = expansion_size(p) if fixed_k is None else fixed_k
             k = min(k, V - 1)
             for r, tok in enumerate(expansion_set(order, k), start=1):

@@ -56,6 +56,11 @@ _SIG = {
     "glide_validate_tree": (ctypes.c_int, [_P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
     "glide_read_device_status": (ctypes.c_int, [_P, _P]),
     "glide_selftest_wait_timeout": (ctypes.c_int, [_P, ctypes.c_uint32, _P]),
+    "glide_cape_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
+    "cape_expand": (ctypes.c_int, [_P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                   ctypes.c_int32, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "glide_kv_compact": (ctypes.c_int, [ctypes.POINTER(AttnDesc), ctypes.c_int32, ctypes.c_int64, _P, _P, _P,
+                                        ctypes.c_int32, _P, _P, _P, _P]),
 }
 
 
@@ -199,6 +204,59 @@ def tree_accept(draft_tokens: torch.Tensor, parent_idx: torch.Tensor, target_log
                            workspace.numel() * workspace.element_size(), _stream(stream))
     _check(st, "tree_accept")
     return path, length, bonus
+
+
+def glide_cape_workspace_bytes(B: int, gamma: int, V: int) -> int:
+    return int(lib().glide_cape_workspace_bytes(B, gamma, V))
+
+
+def cape_expand(probs: torch.Tensor, root_token: torch.Tensor, max_tokens: int, draft_tokens: torch.Tensor,
+                parent_idx: torch.Tensor, n_nodes: torch.Tensor, workspace: torch.Tensor,
+                conf: Optional[torch.Tensor] = None, fixed_k: int = -1, stream=None):
+    """(draft_tokens, parent_idx [B, 1+max_tokens], n_nodes [B]) int32 (and conf [B, gamma] fp32)
+    <- CaPE expansion of the draft distributions probs [B, gamma, V] fp32."""
+    if probs.dim() != 3 or probs.dtype != torch.float32 or not probs.is_contiguous():
+        raise TypeError("probs must be contiguous fp32 [B, gamma, V]")
+    B, gamma, V = probs.shape
+    n_out = 1 + int(max_tokens)
+    for t, shp in ((root_token, (B,)), (draft_tokens, (B, n_out)), (parent_idx, (B, n_out)), (n_nodes, (B,))):
+        if t.dtype != torch.int32 or tuple(t.shape) != shp or not t.is_contiguous():
+            raise TypeError("root, token, parent and count tensors must be contiguous int32 of the stated shapes")
+    if conf is not None and (conf.dtype != torch.float32 or tuple(conf.shape) != (B, gamma)
+                             or not conf.is_contiguous()):
+        raise TypeError("conf must be contiguous fp32 [B, gamma]")
+    st = lib().cape_expand(probs.data_ptr(), root_token.data_ptr(), B, gamma, V, int(max_tokens), int(fixed_k),
+                           draft_tokens.data_ptr(), parent_idx.data_ptr(), n_nodes.data_ptr(),
+                           conf.data_ptr() if conf is not None else None, workspace.data_ptr(),
+                           workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(st, "cape_expand")
+    return draft_tokens, parent_idx, n_nodes
+
+
+def glide_kv_compact(K_cache: torch.Tensor, V_cache: torch.Tensor, kv_len: torch.Tensor, path: torch.Tensor,
+                     length: torch.Tensor, new_kv_len: torch.Tensor, stream=None) -> torch.Tensor:
+    """In-place cache update after acceptance.  K_cache/V_cache are one layer
+    [B, H, S_cap, D] or a stack [layers, B, H, S_cap, D] (contiguous)."""
+    if K_cache.shape != V_cache.shape or K_cache.dtype != V_cache.dtype:
+        raise ValueError("K and V caches must match")
+    if not (K_cache.is_contiguous() and V_cache.is_contiguous()):
+        raise ValueError("caches must be contiguous")
+    if K_cache.dim() == 4:
+        layers, (B, H, S_cap, D) = 1, K_cache.shape
+    elif K_cache.dim() == 5:
+        layers, B, H, S_cap, D = K_cache.shape
+    else:
+        raise ValueError("caches must be [B, H, S_cap, D] or [layers, B, H, S_cap, D]")
+    n = path.shape[-1]
+    for t, shp in ((kv_len, (B,)), (path, (B, n)), (length, (B,)), (new_kv_len, (B,))):
+        if t.dtype != torch.int32 or tuple(t.shape) != shp or not t.is_contiguous():
+            raise TypeError("kv_len, path, len and new_kv_len must be contiguous int32 of the stated shapes")
+    desc = make_desc(B, H, D, S_cap, _dtype_code(K_cache))
+    st = lib().glide_kv_compact(ctypes.byref(desc), layers, B * H * S_cap * D, K_cache.data_ptr(),
+                                V_cache.data_ptr(), kv_len.data_ptr(), n, path.data_ptr(), length.data_ptr(),
+                                new_kv_len.data_ptr(), _stream(stream))
+    _check(st, "glide_kv_compact")
+    return new_kv_len
 
 
 def glide_validate_tree(parent_idx_host, require_root0: bool = True) -> int:

@@ -93,6 +93,11 @@ size_t glide_accept_workspace_bytes(int32_t B, int32_t n) {
   return glide::accept_workspace_bytes(B, n);
 }
 
+size_t glide_cape_workspace_bytes(int32_t B, int32_t gamma, int32_t V) {
+  if (B < 1 || gamma < 1 || gamma > glide::kMaxTree - 1 || V < 1) return 0;
+  return glide::cape_workspace_bytes(B, gamma, V);
+}
+
 glide_status glide_cross_attn(const glide_attn_desc* desc, const void* q_draft, const void* K_cache,
                               const void* V_cache, const int32_t* kv_len, int32_t max_kv_len, float* out,
                               void* workspace, size_t workspace_bytes, glide_stream_t stream) {
@@ -143,6 +148,52 @@ glide_status tree_accept(const int32_t* draft_tokens, const int32_t* parent_idx,
   a.draft = draft_tokens; a.parent = parent_idx; a.logits = target_logits;
   a.B = B; a.n = n; a.V = V; a.path = path; a.len = len; a.bonus = bonus; a.ws = workspace;
   return from_cuda(glide::launch_tree_accept(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+glide_status cape_expand(const float* probs, const int32_t* root_token, int32_t B, int32_t gamma, int32_t V,
+                         int32_t max_tokens, int32_t fixed_k, int32_t* draft_tokens, int32_t* parent_idx,
+                         int32_t* n_nodes, float* conf, void* workspace, size_t workspace_bytes,
+                         glide_stream_t stream) {
+  if (B < 1 || gamma < 1 || V < 1) return GLIDE_ERR_INVALID;
+  if (max_tokens < gamma || max_tokens > glide::kMaxTree - 1) return GLIDE_ERR_INVALID;
+  if (fixed_k < -1) return GLIDE_ERR_INVALID;
+  if (fixed_k > glide::kCapeMaxSet) return GLIDE_ERR_UNSUPPORTED;
+  if (!probs || !root_token || !draft_tokens || !parent_idx || !n_nodes || !workspace) return GLIDE_ERR_INVALID;
+  if (!aligned16(probs) || !aligned16(workspace) || (reinterpret_cast<uintptr_t>(root_token) & 3u) ||
+      (reinterpret_cast<uintptr_t>(draft_tokens) & 3u) || (reinterpret_cast<uintptr_t>(parent_idx) & 3u) ||
+      (reinterpret_cast<uintptr_t>(n_nodes) & 3u) || (reinterpret_cast<uintptr_t>(conf) & 3u))
+    return GLIDE_ERR_INVALID;
+  if (workspace_bytes < glide::cape_workspace_bytes(B, gamma, V)) return GLIDE_ERR_INVALID;
+  glide::CapeArgs a;
+  a.probs = probs; a.root = root_token; a.B = B; a.gamma = gamma; a.V = V;
+  a.max_tokens = max_tokens; a.fixed_k = fixed_k;
+  a.tokens = draft_tokens; a.parent = parent_idx; a.n_nodes = n_nodes; a.conf = conf; a.ws = workspace;
+  return from_cuda(glide::launch_cape_expand(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int64_t layer_stride, void* K_cache,
+                              void* V_cache, const int32_t* kv_len, int32_t n, const int32_t* path,
+                              const int32_t* len, int32_t* new_kv_len, glide_stream_t stream) {
+  if (!desc_ok(desc)) return GLIDE_ERR_INVALID;
+  if (n < 1 || n > glide::kMaxTree || n > desc->S_cap) return GLIDE_ERR_INVALID;
+  if (n_layers < 1) return GLIDE_ERR_INVALID;
+  const int64_t layer_elems = (int64_t)desc->B * desc->H * desc->S_cap * desc->D;
+  if (n_layers > 1 && layer_stride < layer_elems) return GLIDE_ERR_INVALID;
+  if ((double)n_layers * (double)(n_layers > 1 ? layer_stride : layer_elems) > 4.0e18) return GLIDE_ERR_INVALID;
+  const int elt = desc->dtype == GLIDE_BF16 ? 2 : 4;
+  if (n_layers > 1 && ((layer_stride * elt) & 15)) return GLIDE_ERR_INVALID;
+  if (!K_cache || !V_cache || !kv_len || !path || !len || !new_kv_len) return GLIDE_ERR_INVALID;
+  if (!aligned16(K_cache) || !aligned16(V_cache) || (reinterpret_cast<uintptr_t>(kv_len) & 3u) ||
+      (reinterpret_cast<uintptr_t>(path) & 3u) || (reinterpret_cast<uintptr_t>(len) & 3u) ||
+      (reinterpret_cast<uintptr_t>(new_kv_len) & 3u))
+    return GLIDE_ERR_INVALID;
+  if (new_kv_len == kv_len) return GLIDE_ERR_INVALID;
+  glide::CompactArgs a;
+  a.K = K_cache; a.V = V_cache; a.kv_len = kv_len; a.path = path; a.len = len; a.new_kv_len = new_kv_len;
+  a.layers = n_layers; a.layer_stride = n_layers > 1 ? layer_stride : layer_elems;
+  a.B = desc->B; a.H = desc->H; a.D = desc->D; a.S_cap = desc->S_cap; a.n = n;
+  a.dtype = desc->dtype == GLIDE_BF16 ? 0 : 1;
+  return from_cuda(glide::launch_kv_compact(a, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 glide_status glide_validate_tree(const int32_t* parent_idx_host, int32_t B, int32_t n, int32_t require_root0) {

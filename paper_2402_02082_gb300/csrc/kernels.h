@@ -9,6 +9,7 @@ namespace glide {
 constexpr int kMaxBatch = 1024;   // sequences per call (per-CTA tile table lives in shared memory)
 constexpr int kMaxTree = 64;      // tree nodes (one 64-bit ancestor mask per node)
 constexpr int kMaxCtas = 1024;    // CTAs per attention launch (bounds the partial slots)
+constexpr int kCapeMaxSet = 7;    // largest expansion set: S(p) <= 7, fixed sizes up to 7
 
 struct AttnArgs {
   const void* q;
@@ -38,6 +39,32 @@ struct AcceptArgs {
   void* ws;
 };
 
+struct CapeArgs {
+  const float* probs;     // [B, gamma, V]
+  const int32_t* root;    // [B]
+  int B, gamma, V;
+  int max_tokens;         // gamma .. kMaxTree - 1
+  int fixed_k;            // -1: S(p); else 0 .. kCapeMaxSet
+  int32_t* tokens;        // [B, 1 + max_tokens]
+  int32_t* parent;        // [B, 1 + max_tokens]
+  int32_t* n_nodes;       // [B]
+  float* conf;            // [B, gamma] or null
+  void* ws;
+};
+
+struct CompactArgs {
+  void* K;
+  void* V;
+  const int32_t* kv_len;
+  const int32_t* path;
+  const int32_t* len;
+  int32_t* new_kv_len;
+  int layers;
+  long long layer_stride;  // elements between layers
+  int B, H, D, S_cap, n;
+  int dtype;               // 0 bf16, 1 f32
+};
+
 int sm_count();  // multiprocessors of the current device (cached per device)
 
 cudaError_t launch_cross_attn(const AttnArgs& a, cudaStream_t st);
@@ -46,6 +73,10 @@ cudaError_t launch_tree_attn_fma(const AttnArgs& a, cudaStream_t st);
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st);
 cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st);
 
+cudaError_t launch_cape_expand(const CapeArgs& a, cudaStream_t st);
+cudaError_t launch_kv_compact(const CompactArgs& a, cudaStream_t st);
+
 size_t accept_workspace_bytes(int B, int n);
+size_t cape_workspace_bytes(int B, int gamma, int V);
 
 }  // namespace glide

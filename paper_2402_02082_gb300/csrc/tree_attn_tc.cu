@@ -24,8 +24,10 @@
 //              the halves are merged once per segment.  Query i sits in row
 //              (i % 4) * 16 + i / 4, which spreads any tree over all four lane
 //              quarters (all four SM sub-partitions).
-//   warp 8     producer: lane 0 loads K tiles, lane 1 V tiles, with 2-D TMA
-//              (64 keys x 64 head dims per box, 128-byte swizzle).
+//   warp 8     producer: lane 0 feeds both the K and the V ring with 2-D TMA
+//              (64 keys x 64 head dims per box, 128-byte swizzle), polling
+//              both rings' free slots without blocking on either (K slots free
+//              up after S, V slots only after P.V).
 //   warps 9-11 MMA issue.  A tcgen05.mma keeps its issuing thread busy for
 //              ~150 cycles whatever its shape, so one thread cannot feed a
 //              64-key tile (8 S + 4 P.V instructions) at HBM speed: warp 9

@@ -165,7 +165,8 @@ def draft_probs(seed: int, B: int, gamma: int, vocab: int, quantum: float = 0.0)
         for i in range(gamma):
             conf = g.uniform(0.05, 0.98)
             tail = g.gamma(0.3, size=vocab - 1)
-            tail *= (1.0 - conf) / tail.sum()
+            if vocab > 1:
+                tail *= (1.0 - conf) / tail.sum()
             tail = np.minimum(tail, conf)
             row = np.insert(tail, int(g.integers(vocab)), conf)
             if quantum > 0:

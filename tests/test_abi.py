@@ -102,6 +102,32 @@ def test_accept_rejects(L):
         assert acc(**b) == gb.GLIDE_ERR_INVALID, b
 
 
+def test_cape_rejects(L):
+    assert gb.glide_cape_workspace_bytes(4, 5, 32000) > 0
+    for b in ((0, 5, 10), (4, 0, 10), (4, 64, 10), (4, 5, 0)):
+        assert gb.glide_cape_workspace_bytes(*b) == 0, b
+
+    def cape(probs=FAKE, root=FAKE, B=2, gamma=5, V=1000, max_tokens=32, fixed_k=-1, tok=FAKE, par=FAKE,
+             nn=FAKE, conf=None, ws=FAKE, wsb=1 << 30):
+        return L.cape_expand(probs, root, B, gamma, V, max_tokens, fixed_k, tok, par, nn, conf, ws, wsb, None)
+    for b in [dict(B=0), dict(gamma=0), dict(V=0), dict(max_tokens=4), dict(max_tokens=64), dict(fixed_k=-2),
+              dict(probs=None), dict(root=None), dict(tok=None), dict(par=None), dict(nn=None), dict(ws=None),
+              dict(wsb=64), dict(probs=FAKE + 4), dict(ws=FAKE + 8), dict(tok=FAKE + 2), dict(conf=FAKE + 1)]:
+        assert cape(**b) == gb.GLIDE_ERR_INVALID, b
+    assert cape(fixed_k=8) == gb.GLIDE_ERR_UNSUPPORTED
+
+
+def test_kv_compact_rejects(L):
+    def comp(d=None, layers=1, stride=0, K=FAKE, V=FAKE, kv=FAKE, n=5, path=FAKE, ln=FAKE, new=FAKE + 256):
+        d = d or desc()
+        return L.glide_kv_compact(ctypes.byref(d), layers, stride, K, V, kv, n, path, ln, new, None)
+    elems = 2 * 4 * 300 * 128
+    for b in [dict(n=0), dict(n=65), dict(layers=0), dict(layers=2, stride=elems - 1), dict(layers=2, stride=elems + 4),
+              dict(K=None), dict(V=None), dict(kv=None), dict(path=None), dict(ln=None), dict(new=None),
+              dict(K=FAKE + 8), dict(path=FAKE + 2), dict(new=FAKE), dict(d=desc(D=80)), dict(d=desc(S_cap=4))]:
+        assert comp(**b) == gb.GLIDE_ERR_INVALID, b
+
+
 def test_validate_tree(L):
     assert gb.glide_validate_tree(np.array([-1, 0, 1, 1, 0])) == gb.GLIDE_OK
     assert gb.glide_validate_tree(np.array([[-1, 0, 0], [-1, 0, 1]])) == gb.GLIDE_OK
