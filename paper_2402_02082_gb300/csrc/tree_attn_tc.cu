@@ -90,7 +90,7 @@ struct TcCfg {
   static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKVTile; }
   static __host__ __device__ uint32_t off_ml(int ns) { return off_bar(ns) + 512; }
   static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + kM * 8; }
-  static __host__ __device__ uint32_t off_tab(int ns) { return off_misc(ns) + 32; }
+  static __host__ __device__ uint32_t off_tab(int ns) { return off_misc(ns) + 48; }
   static constexpr uint32_t kTmemO = kSBuf * kTK;                  // S buffers at columns 0, 64, 128, 192
   static constexpr uint32_t kTmemCols = kTmemO + 2 * D <= 256 ? 256 : 512;
   static_assert(kTmemO + 2 * D <= 512, "TMEM columns");
@@ -132,6 +132,12 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 // Named barrier among the 256 softmax threads (id 2; id 1 belongs to the split merge).
 __device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
+// Barrier 3 hands the (max, sum) exchange slot back from the key-half-0 warps
+// (arrive, after reading it) to the key-half-1 warps (sync, before writing it
+// for the next segment).  Both sides count the same segments, so every sync
+// has its arrivals.
+__device__ __forceinline__ void ml_release() { asm volatile("bar.arrive 3, 256;" ::: "memory"); }
+__device__ __forceinline__ void ml_acquire() { asm volatile("bar.sync 3, 256;" ::: "memory"); }
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -147,6 +153,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
   volatile int* last_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 8);
+  int* pend_count = reinterpret_cast<int*>(base + C::off_misc(ns) + 12);
+  int4* pend = reinterpret_cast<int4*>(base + C::off_misc(ns) + 16);  // at most 2 split segments
   BatchTiles bt;
   bt.start = reinterpret_cast<long long*>(base + C::off_tab(ns));
   bt.len = reinterpret_cast<int*>(bt.start + p.B + 1);
@@ -163,6 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars[b], cnt);
     }
     *abort_flag = 0;
+    *pend_count = 0;
     fence_barrier_init();
   }
   if (warp == kMmaWarp) {
@@ -331,30 +340,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int sid = threadIdx.x;                  // 0..255 among the softmax threads
     const float sl2 = p.scale_log2;
     bool dead = false;
-    int i = 0, seg = 0;
+    int i = 0, seg = 0, npend = 0;
+    // Segment sg's queries into the swizzled Q tile (padding rows are zero);
+    // the two threads of a row write chunks 0-3 and 4-7 of each 128-byte atom.
+    // Key-half-0 warps only.
+    auto write_q = [&](const Segment& sq, int sg) {
+      unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
+      const uint4* src =
+          reinterpret_cast<const uint4*>(p.q + (((size_t)sq.b * n + (valid ? qi : 0)) * p.H + sq.h) * D);
+#pragma unroll
+      for (int hd = 0; hd < C::kHalves; ++hd)
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+          const int c = cpar * 4 + cc;
+          uint4 v = make_uint4(0u, 0u, 0u, 0u);
+          if (valid) v = src[hd * 8 + c];
+          *reinterpret_cast<uint4*>(qrow + hd * C::kQHalf + ((c ^ (row & 7)) << 4)) = v;
+        }
+      tc::fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_QFULL + (sg & 1)]);
+    };
     for (long long g = g_begin; g < g_end; ++seg) {
       const Segment s = locate(bt, P, p.B, g, g_end);
       const int plen = bt.plen[s.b], len = bt.len[s.b];
 
-      if (half == 0) {
-        // this segment's queries into the swizzled Q tile (padding rows are zero);
-        // the two threads of a row write chunks 0-3 and 4-7 of each 128-byte atom
-        unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
-        const uint4* src =
-            reinterpret_cast<const uint4*>(p.q + (((size_t)s.b * n + (valid ? qi : 0)) * p.H + s.h) * D);
-#pragma unroll
-        for (int hd = 0; hd < C::kHalves; ++hd)
-#pragma unroll
-          for (int cc = 0; cc < 4; ++cc) {
-            const int c = cpar * 4 + cc;
-            uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (valid) v = src[hd * 8 + c];
-            *reinterpret_cast<uint4*>(qrow + hd * C::kQHalf + ((c ^ (row & 7)) << 4)) = v;
-          }
-        tc::fence_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars[B_QFULL + (seg & 1)]);
-      }
+      if (half == 0 && seg == 0) write_q(s, 0);  // later segments' Q is written ahead (below)
       uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
       if (valid) {
         int j = qi;
@@ -484,14 +495,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bars[B_PFULL + (j & 1)]);
       }
 
+      // Every S product of this segment has been consumed, so Q is free: write
+      // the next segment's queries now and let its S products overlap this
+      // epilogue.
+      if (half == 0 && s.g_end < g_end) write_q(locate(bt, P, p.B, s.g_end, g_end), seg + 1);
+
       // ---- segment epilogue: merge the two key halves, then O / l or a split partial
       l += __shfl_xor_sync(0xffffffffu, l, 2);  // the row's sum over both threads
-      if (half == 1 && cpar == 0) ml[row] = make_float2(m_used, l);
+      if (half == 1) {
+        // the next segment's Q is written ahead, so these warps can reach this
+        // point again while the half-0 warps still read the slot
+        if (seg > 0) ml_acquire();
+        if (cpar == 0) ml[row] = make_float2(m_used, l);
+      }
       softmax_sync();
       if (half == 0) {
         const int jl = i - 1;
         if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 3)], (jl >> 2) & 1, abort_flag, p.status);
         const float2 other = ml[row];
+        if (s.g_end < g_end) ml_release();
         const float M = fmaxf(m_used, other.x);
         const float f0 = m_used == -CUDART_INF_F ? 0.f : fast_exp2(m_used - M);
         const float f1 = other.x == -CUDART_INF_F ? 0.f : fast_exp2(other.x - M);
@@ -510,10 +532,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + c * 32, a);
             tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + D + c * 32, b);
             tc::tmem_wait_ld();
-            if (valid) {
+            float v[16];
 #pragma unroll
-              for (int k = 0; k < 16; ++k)
-                dst[c * 32 + 2 * k + cpar] = __uint_as_float(a[k]) * g0 + __uint_as_float(b[k]) * g1;
+            for (int k = 0; k < 16; ++k) v[k] = __uint_as_float(a[k]) * g0 + __uint_as_float(b[k]) * g1;
+            // The row's two threads hold its even (cpar 0) and odd (cpar 1)
+            // columns; one exchange of two values per 8 columns gives each
+            // thread 4 consecutive columns: cpar 0 columns 8j..8j+3, cpar 1
+            // columns 8j+4..8j+7.
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const float r0 = __shfl_xor_sync(0xffffffffu, cpar ? v[4 * j] : v[4 * j + 2], 2);
+              const float r1 = __shfl_xor_sync(0xffffffffu, cpar ? v[4 * j + 1] : v[4 * j + 3], 2);
+              const float4 q4 = cpar ? make_float4(r0, v[4 * j + 2], r1, v[4 * j + 3])
+                                     : make_float4(v[4 * j], r0, v[4 * j + 1], r1);
+              float* d4 = dst + c * 32 + 8 * j + 4 * cpar;
+              if (valid) {
+                if (single) {
+                  *reinterpret_cast<float4*>(d4) = q4;
+                } else {  // a partial row starts 8 bytes into a 16-byte boundary
+                  reinterpret_cast<float2*>(d4)[0] = make_float2(q4.x, q4.y);
+                  reinterpret_cast<float2*>(d4)[1] = make_float2(q4.z, q4.w);
+                }
+              }
             }
           }
           if (!single && valid && cpar == 0) {
@@ -524,10 +564,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars[B_OFREE]);
-        if (!single) combine_if_last(s, p.B, p.H, n, D, p.partials, p.counters, p.out, threadIdx.x, 128, last_flag);
+        // A split (b, h) is merged by the CTA that completes its count, but only
+        // after this CTA's last tile (see the end of the kernel), so that the
+        // merge does not hold up the next segment.  Only the first and the last
+        // segment of a CTA's share can be split.
+        if (!single && arrive_split(s, p.H, p.counters, threadIdx.x, 128, last_flag)) {
+          if (sid == 0) pend[npend] = make_int4(s.b, s.h, s.c_first, s.c_last);
+          ++npend;
+        }
       }
       g = s.g_end;
     }
+    if (sid == 0) pend_count[0] = npend;
   }
 
   __syncwarp();  // the producer and MMA warps reconverge after their single-lane loops
@@ -536,6 +584,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kMmaWarp) {
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, C::kTmemCols);
+  }
+  // The split (b, h) this CTA completed, merged by all threads (no waiting,
+  // so also after an abort: the counters are re-armed either way); the P
+  // buffers, which no MMA reads any more, are the scratch.
+  const int np = pend_count[0];
+  for (int k = 0; k < np; ++k) {
+    Segment s;
+    s.b = pend[k].x; s.h = pend[k].y; s.c_first = pend[k].z; s.c_last = pend[k].w;
+    combine_partials(s, p.H, n, D, p.partials, p.counters, p.out, reinterpret_cast<float*>(base + C::off_P),
+                     threadIdx.x, kThreads);
   }
 }
 
