@@ -246,6 +246,8 @@ def workload_config(w):
 
 
 # -------------------------------------------------------------------- main
+# kernels each library call launches (cross-attention: the attention kernel and its merge)
+LAUNCHES_PER_CALL = {"glide_cross_attn": 2, "tree_verify_attn": 1, "tree_accept": 1}
 CAPE_MAX_TOKENS = 32   # the cap on verified tokens of the paper's CaPE runs (Section 4)
 
 
@@ -547,7 +549,7 @@ def run_glide(args, rank, world, local_rank):
                 "roofline": roof, "kernels": kernels, "next_rows": next_rows, "cpu_baseline": cpu_baseline,
                 "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                         "steps": e2e_steps},
-                "gpu_launches": len(step_fns) * args.steps, "clocks": clk}
+                "gpu_launches": sum(LAUNCHES_PER_CALL[nm] for nm in names) * args.steps, "clocks": clk}
         if args.force_fma:
             line["config"]["tree_kernel"] = "cuda-core (forced)"
         print(json.dumps(line))

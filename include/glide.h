@@ -236,11 +236,11 @@ glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int
  * host engine owns and budgets all device memory, or a serving loop that has
  * given nearly all of HBM to its KV cache and bans allocator calls on its
  * per-token path.  Same arguments and result as glide_cross_attn, minus the
- * workspace: the scratch lives in one fixed 4 MiB array inside the library,
+ * workspace: the scratch lives in one fixed 32 MiB array inside the library,
  * held on every GPU that loads the library until the process exits.
  * - Shapes whose workspace (glide_attn_workspace_bytes(desc, 1)) exceeds
- *   4 MiB are rejected with GLIDE_ERR_UNSUPPORTED (B*H up to 6987 for D = 128,
- *   14640 for D = 64).
+ *   32 MiB are rejected with GLIDE_ERR_UNSUPPORTED (B*H up to 7035 for D = 128,
+ *   14835 for D = 64).
  * - The first call on each device looks up the array's device address; make
  *   that first call before any stream capture.
  * - Every call first clears the words that must start at zero, then reuses the

@@ -47,8 +47,11 @@ bool desc_ok(const glide_attn_desc* d) {
 }
 
 size_t attn_ws_bytes(const glide_attn_desc* d, int nq) {
+  // partial slots: one per (share or chunk, b, h) pair index; a tree slot holds
+  // nq query rows, a cross-attention slot one row per consumer warp
   const size_t slots = (size_t)glide::kMaxCtas + (size_t)d->B * d->H;
-  return glide::WsLayout::partials_off(d->B, d->H) + slots * (size_t)nq * (d->D + 2) * sizeof(float);
+  const size_t rows = (size_t)(nq > glide::kCrossPartials ? nq : glide::kCrossPartials);
+  return glide::WsLayout::partials_off(d->B, d->H) + slots * rows * (d->D + 2) * sizeof(float);
 }
 
 glide::AttnArgs make_args(const glide_attn_desc* d, const void* q, const void* K, const void* V,

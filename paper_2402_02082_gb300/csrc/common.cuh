@@ -14,14 +14,22 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull; // 1 s: far beyond any legitima
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ---------------------------------------------------------------- workspace
-// Attention workspace: [0,256) status word; [256, 256 + 4*B*H) per-(b,h)
-// arrival counters; then 256-aligned partial slots of nq*(D+2) floats.
+// Attention workspace: [0,256) header (the status word at byte 0; the
+// cross-attention chunk-claim counter at byte 128 and its CTA-done counter at
+// byte 192); then per-(b,h) arrival counters (4 bytes each, tree kernels);
+// then per-(b,h) chunk ranges (8 bytes each, cross-attention scratch); then
+// 256-aligned partial slots of nq*(D+2) floats.
 struct WsLayout {
   static constexpr size_t kHeader = 256;
+  static constexpr size_t kClaimOff = 128;
+  static constexpr size_t kDoneOff = 192;
+  static __host__ __device__ size_t align(size_t x) { return (x + 255) & ~size_t(255); }
   static __host__ __device__ size_t counters_off() { return kHeader; }
+  static __host__ __device__ size_t ranges_off(int B, int H) {
+    return align(kHeader + sizeof(unsigned) * (size_t)B * H);
+  }
   static __host__ __device__ size_t partials_off(int B, int H) {
-    size_t c = kHeader + sizeof(unsigned) * (size_t)B * H;
-    return (c + 255) & ~size_t(255);
+    return align(ranges_off(B, H) + 2 * sizeof(int) * (size_t)B * H);
   }
 };
 
@@ -194,6 +202,54 @@ __device__ inline void build_batch_tiles(BatchTiles bt, const int* kv_len, int B
   __syncthreads();
 }
 
+// Dynamic work: the global tile sequence is cut into chunks of shrinking size
+// that CTAs claim at run time.  Level 0 holds the first half of the tiles in
+// G equal chunks, level 1 half of the rest in G chunks, and so on; the last
+// level takes what remains.  The big early chunks keep claims few; the small
+// late ones let the CTAs that stream faster take more of the work, so all of
+// them finish close together.  Levels are dropped until every level has at
+// least G tiles, so an empty chunk (tiles < G, one level) can only sit at
+// the very end of the sequence, never inside a (b, h).  cta_of() names the
+// chunk that holds a tile, which is what the split-merge bookkeeping needs.
+constexpr int kMaxLevels = 6;
+struct Chunks {
+  long long lo[kMaxLevels + 1];
+  int G, L;
+  __device__ void init(long long total, int grid, int levels) {
+    G = grid;
+    L = levels < 1 ? 1 : (levels > kMaxLevels ? kMaxLevels : levels);
+    for (;; --L) {
+      long long a = 0;
+      bool ok = true;
+      for (int l = 0; l < L; ++l) {
+        lo[l] = a;
+        const long long size = (l == L - 1) ? total - a : (total - a) / 2;
+        if (size < G) ok = false;
+        a += size;
+      }
+      lo[L] = total;
+      if (ok || L == 1) break;
+    }
+  }
+  __device__ int count() const { return G * L; }
+  __device__ long long begin(int k) const {
+    const int l = k / G, j = k - l * G;
+    if (l >= L) return lo[L];
+    const long long size = lo[l + 1] - lo[l], base = size / G, rem = size % G;
+    return lo[l] + (long long)j * base + (j < rem ? j : rem);
+  }
+  __device__ long long end(int k) const { return begin(k + 1); }
+  __device__ int cta_of(long long g) const {
+    int l = 0;
+    while (l + 1 < L && g >= lo[l + 1]) ++l;
+    const long long size = lo[l + 1] - lo[l], base = size / G, rem = size % G;
+    const long long off = g - lo[l];
+    const long long big = rem * (base + 1);
+    const long long j = off < big ? off / (base + 1) : rem + (off - big) / base;
+    return l * G + (int)j;
+  }
+};
+
 struct Segment {
   int b, h;
   int t0, t1;          // tile range within the (b, h) slab, [t0, t1)
@@ -201,9 +257,11 @@ struct Segment {
   int c_first, c_last; // CTAs that share this (b, h)
 };
 
-// Locates the segment that starts at global tile g (< g_limit, the CTA's end).
-__device__ inline Segment locate(const BatchTiles& bt, const Partition& P, int B, long long g,
-                                 long long g_limit) {
+// Locates the segment that starts at global tile g (< g_limit, the end of the
+// CTA's share or chunk).  Part is Partition or Chunks: c_first / c_last name
+// the shares (chunks) that hold the (b, h)'s first and last tile.
+template <class Part>
+__device__ inline Segment locate(const BatchTiles& bt, const Part& P, int B, long long g, long long g_limit) {
   int lo = 0, hi = B - 1;  // last b with start[b] <= g
   while (lo < hi) {
     int mid = (lo + hi + 1) >> 1;

@@ -24,7 +24,7 @@
 
 namespace {
 
-constexpr size_t kScratchBytes = 4u << 20;  // 4 MiB per GPU
+constexpr size_t kScratchBytes = 32u << 20;  // 32 MiB per GPU
 constexpr int kMaxDevices = 64;
 
 // The scratch itself.  In host code this name is only a host-side stand-in
