@@ -207,11 +207,14 @@ __device__ inline void build_batch_tiles(BatchTiles bt, const int* kv_len, int B
 // G equal chunks, level 1 half of the rest in G chunks, and so on; the last
 // level takes what remains.  The big early chunks keep claims few; the small
 // late ones let the CTAs that stream faster take more of the work, so all of
-// them finish close together.  Levels are dropped until every level has at
-// least G tiles, so an empty chunk (tiles < G, one level) can only sit at
-// the very end of the sequence, never inside a (b, h).  cta_of() names the
-// chunk that holds a tile, which is what the split-merge bookkeeping needs.
+// them finish close together.  Levels are dropped until every chunk of every
+// level has at least kMinChunk tiles (fewer, smaller chunks only add partial
+// results to merge) or one level is left; with one level an empty chunk
+// (tiles < G) can only sit at the very end of the sequence, never inside a
+// (b, h).  cta_of() names the chunk that holds a tile, which is what the
+// split-merge bookkeeping needs.
 constexpr int kMaxLevels = 6;
+constexpr long long kMinChunk = 16;
 struct Chunks {
   long long lo[kMaxLevels + 1];
   int G, L;
@@ -224,7 +227,7 @@ struct Chunks {
       for (int l = 0; l < L; ++l) {
         lo[l] = a;
         const long long size = (l == L - 1) ? total - a : (total - a) / 2;
-        if (size < G) ok = false;
+        if (size < G * kMinChunk) ok = false;
         a += size;
       }
       lo[L] = total;

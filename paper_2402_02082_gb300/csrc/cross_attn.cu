@@ -335,14 +335,14 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
 // Merges, for each (b, h), the partials of every consumer warp of every chunk
 // that holds part of its keys (slots (c + b*H + h) * 8 + w for c in its chunk
 // range): out = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s.  One CTA per
-// (b, h) (a (b, h) in the small late chunks has ~200 partials): threads
-// stride over the partials for M and the sum, then each warp takes every
-// eighth partial, lanes owning D / 32 consecutive columns, with a group of
-// partials' loads issued before any use; the warps' sums meet in shared
-// memory.  A warp that had no tile of a segment left max = -inf and no o: its
+// (b, h) (a (b, h) in the small late chunks has a few hundred partials):
+// threads stride over the partials for M and the sum, then each of the 16
+// warps takes every 16th partial, lanes owning D / 32 consecutive columns,
+// with a group of 8 partials' loads issued before any use; the warps' sums
+// meet in shared memory.  A warp that had no tile of a segment left max = -inf and no o: its
 // weight is 0 and its o never reaches a sum.
-constexpr int kMergeWarps = 8;
-constexpr int kMergeGroup = 4;  // partials per warp whose loads are issued together
+constexpr int kMergeWarps = 16;
+constexpr int kMergeGroup = 8;  // partials per warp whose loads are issued together
 template <int D>
 __global__ void __launch_bounds__(kMergeWarps * 32) cross_merge_kernel(const int2* ranges, const float* partials,
                                                                       float* out, int BH) {
