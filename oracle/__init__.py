@@ -20,6 +20,9 @@ It is a plain, slow, fp64 restatement of what the path computes:
   sized expansion sets, and the linearized token tree.
 * ``kvcache.kv_compact``         -- the cache update after verification
   (Section 3.1): the accepted path's entries become contiguous rows.
+* ``sampling.spec_sample_accept`` -- speculative-sampling acceptance of a
+  chain proposal (the strategy Section 2 names and Section 4.1 uses for GliDe
+  alone), with the random numbers as inputs.
 
 Every function here is pinned by tests in ``tests/test_oracle.py`` against
 closed forms, library routines, brute force and invariants; none is marked
@@ -30,6 +33,8 @@ from .attention import (ancestors_or_self, cape_mask, cross_attn, tree_allowed_m
 from .accept import row_argmax, tree_accept
 from .cape import cape_expand, expansion_size
 from .kvcache import kv_compact
+from .sampling import spec_sample_accept
 
 __all__ = ["ancestors_or_self", "cape_mask", "cross_attn", "tree_allowed_mask",
-           "tree_verify_attn", "widen", "row_argmax", "tree_accept", "cape_expand", "expansion_size", "kv_compact"]
+           "tree_verify_attn", "widen", "row_argmax", "tree_accept", "cape_expand", "expansion_size", "kv_compact",
+           "spec_sample_accept"]

@@ -585,3 +585,108 @@ def check_kv_compact_chain_identity(kv_compact):
     K2, V2, nl = kv_compact(K, V, [3, 10], path, [2, 5])
     assert np.array_equal(K2, K) and np.array_equal(V2, V)
     assert list(nl) == [6, 16]
+
+
+# ------------------------------------------------- speculative sampling
+def read_spec_sample_golden():
+    ex, cur = [], None
+    for ln in open(os.path.join(GOLDEN, "spec_sample_examples.txt")):
+        ln = ln.strip()
+        if not ln or ln.startswith("#"):
+            continue
+        key, *vals = ln.split()
+        if key == "example":
+            cur = {"name": vals[0], "pt": [], "q": []}
+            ex.append(cur)
+        elif key in ("pt", "q"):
+            cur[key].append([float(v) for v in vals])
+        elif key in ("gamma", "vocab"):
+            cur[key] = int(vals[0])
+        elif key in ("draft", "out"):
+            cur[key] = [int(v) for v in vals]
+        else:
+            cur[key] = [float(v) for v in vals]
+    return ex
+
+
+def spec_golden_arrays(ex):
+    """(draft [1, g], q [1, g, V] fp32, target logits [1, g+1, V] fp32, u [1, g+1] fp32)."""
+    with np.errstate(divide="ignore"):
+        lg = np.log(np.array(ex["pt"], dtype=np.float64))
+    lg = np.where(np.isfinite(lg), lg, -1e4).astype(np.float32)
+    return (np.array([ex["draft"]], dtype=np.int32), np.array([ex["q"]], dtype=np.float32), lg[None],
+            np.array([ex["u"]], dtype=np.float32))
+
+
+def check_spec_sample_golden(spec_sample_accept):
+    for ex in read_spec_sample_golden():
+        n, tok = spec_sample_accept(*spec_golden_arrays(ex))
+        assert [int(n[0]), int(tok[0])] == ex["out"], ex["name"]
+
+
+def _first_token_law(spec_sample_accept, q, logits, grid=2000):
+    """Law of the first emitted token when x_1 ~ q and u, v are uniform, for
+    gamma = 1, measured by running the rule over midpoint grids: the accept
+    probability of each x over a u grid, the residual draw over a v grid."""
+    V = len(q)
+    mid = ((np.arange(grid) + 0.5) / grid).astype(np.float32)
+    law = np.zeros(V)
+    acc_rate = 0.0
+    for x in range(V):
+        if q[x] == 0:
+            continue
+        draft = np.full((grid, 1), x, dtype=np.int32)
+        qs = np.broadcast_to(q, (grid, 1, V)).astype(np.float32)
+        lg = np.broadcast_to(logits, (grid, 2, V)).astype(np.float32)
+        u = np.stack([mid, np.zeros(grid, np.float32)], axis=1)
+        n, _ = spec_sample_accept(draft, qs, lg, u)
+        acc = float(np.mean(n == 1))
+        u_rej = np.stack([np.full(grid, 0.99999994, np.float32), mid], axis=1)
+        n2, tok = spec_sample_accept(draft, qs, lg, u_rej)
+        if acc < 1.0:
+            assert np.all(n2 == 0), "u close to 1 must reject a token the target likes less"
+            resid = np.bincount(tok, minlength=V) / grid
+        else:
+            resid = np.zeros(V)
+        law[x] += q[x] * acc
+        law += q[x] * (1.0 - acc) * resid
+        acc_rate += q[x] * acc
+    return law, acc_rate
+
+
+def check_spec_sample_is_target_sampling(spec_sample_accept):
+    """The defining property of speculative sampling: with x_1 drawn from the
+    draft, the first emitted token is distributed as the target's own sample,
+    and a proposal is accepted with probability sum_x min(p_T(x), p_D(x))
+    (Section 4.1, "Metrics")."""
+    g = _rng(30)
+    for trial in range(6):
+        V = int(g.integers(3, 7))
+        q = g.dirichlet(np.full(V, 0.7)).astype(np.float32)
+        logits = (g.standard_normal((2, V)) * 1.5).astype(np.float32)
+        law, acc_rate = _first_token_law(spec_sample_accept, q, logits)
+        p = np.exp(logits[0].astype(np.float64) - logits[0].max())
+        p /= p.sum()
+        assert np.abs(law - p).max() < 5e-3, f"trial {trial}: law {law} vs target {p}"
+        alpha = np.minimum(p, q.astype(np.float64)).sum()
+        assert abs(acc_rate - alpha) < 5e-3, f"trial {trial}: acceptance {acc_rate} vs {alpha}"
+
+
+def check_spec_sample_same_model_accepts(spec_sample_accept):
+    """A draft equal to the target (up to fp32 rounding) is always accepted
+    for u below 1 - 1e-6, and the extra token is then the inverse-CDF draw
+    from the last target row."""
+    g = _rng(31)
+    B, gamma, V = 40, 5, 50
+    logits = (g.standard_normal((B, gamma + 1, V)) * 2).astype(np.float32)
+    z = logits.astype(np.float64)
+    q = np.exp(z - z.max(-1, keepdims=True))
+    q = (q / q.sum(-1, keepdims=True)).astype(np.float32)[:, :gamma]
+    draft = np.stack([[int(g.choice(V, p=q[b, i] / q[b, i].sum())) for i in range(gamma)] for b in range(B)])
+    u = (g.random((B, gamma + 1)) * 0.999).astype(np.float32)
+    n, tok = spec_sample_accept(draft.astype(np.int32), q, logits, u)
+    assert np.all(n == gamma)
+    for b in range(B):
+        p = np.exp(z[b, gamma] - z[b, gamma].max())
+        c = np.cumsum(p / p.sum())
+        assert int(tok[b]) == int(np.searchsorted(c, float(u[b, gamma]), side="right"))

@@ -324,3 +324,66 @@ def test_mutant_kv_reversed_path():
             rev[b, :m] = path[b, :m][::-1]
         return okv.kv_compact(K, V, kv_len, rev, length)
     _expect_some_fail(_kv_pins(bad))
+
+
+# ------------------------------------------------- speculative sampling
+from oracle import sampling as osamp
+
+
+def test_spec_sample_golden():
+    pins.check_spec_sample_golden(osamp.spec_sample_accept)
+
+
+def test_spec_sample_is_target_sampling():
+    pins.check_spec_sample_is_target_sampling(osamp.spec_sample_accept)
+
+
+def test_spec_sample_same_model_accepts():
+    pins.check_spec_sample_same_model_accepts(osamp.spec_sample_accept)
+
+
+def _sampling_pins():
+    return [lambda: pins.check_spec_sample_golden(osamp.spec_sample_accept),
+            lambda: pins.check_spec_sample_is_target_sampling(osamp.spec_sample_accept),
+            lambda: pins.check_spec_sample_same_model_accepts(osamp.spec_sample_accept)]
+
+
+def test_mutant_sampling_ratio_inverted(monkeypatch):
+    monkeypatch.setattr(osamp, "accepts", lambda u, pd, pt: float(u) * float(pt) < float(pd))
+    _expect_some_fail(_sampling_pins())
+
+
+def test_mutant_sampling_non_strict(monkeypatch):
+    monkeypatch.setattr(osamp, "accepts", lambda u, pd, pt: float(u) * float(pd) <= float(pt))
+    _expect_some_fail(_sampling_pins())
+
+
+def test_mutant_sampling_unclipped_residual(monkeypatch):
+    def unclipped(pt, pd):
+        w = pt - pd.astype(np.float64)
+        return w if w.sum() > 0 else pt
+    monkeypatch.setattr(osamp, "residual_weights", unclipped)
+    _expect_some_fail(_sampling_pins())
+
+
+def test_mutant_sampling_unnormalised_draw(monkeypatch):
+    def raw(w, v):
+        c = np.cumsum(w)
+        idx = int(np.searchsorted(c, float(v), side="right"))
+        return min(idx, len(w) - 1)
+    monkeypatch.setattr(osamp, "inverse_cdf", raw)
+    _expect_some_fail(_sampling_pins())
+
+
+def test_mutant_sampling_bonus_from_last_proposal_row():
+    def bad(draft_tokens, draft_probs, target_logits, uniforms):
+        # the extra token after a full acceptance drawn from p_T,gamma (the last
+        # proposal position) instead of p_T,gamma+1
+        shifted = target_logits.copy()
+        shifted[:, -1] = target_logits[:, -2]
+        n, tok = osamp.spec_sample_accept(draft_tokens, draft_probs, target_logits, uniforms)
+        n2, tok2 = osamp.spec_sample_accept(draft_tokens, draft_probs, shifted, uniforms)
+        gamma = draft_tokens.shape[1]
+        return n, np.where(n == gamma, tok2, tok)
+    _expect_some_fail([lambda: pins.check_spec_sample_golden(bad),
+                       lambda: pins.check_spec_sample_same_model_accepts(bad)])
