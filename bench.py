@@ -311,8 +311,25 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
     e = 2 if w.dtype == "bf16" else 4
     moved = sum(1 for b in range(B) for k in range(1, int(l_h[b]) + 1) if int(p_h[b, k]) != k)
     comp_bytes = moved * w.H * w.D * e * 2 * 2 + B * (4 * 3 + 4 * (int(l_h.max()) + 1))
+    # speculative-sampling acceptance of a gamma-token chain (the GliDe-alone setting)
+    sq = synth.draft_probs(w.seed + 18, B, w.gamma, w.vocab)
+    s_draft = torch.from_numpy(synth.sample_tokens(w.seed + 18, sq)).to(dev)
+    s_logits = torch.from_numpy(synth.target_logits_near(w.seed + 18, sq, 0.7)).to(dev)
+    s_u = torch.from_numpy(synth.uniforms(w.seed + 18, (B, w.gamma + 1))).to(dev)
+    s_q = torch.from_numpy(sq).to(dev)
+    s_n = torch.empty(B, dtype=torch.int32, device=dev)
+    s_t = torch.empty(B, dtype=torch.int32, device=dev)
+    ws_s = torch.zeros(gb.glide_sample_workspace_bytes(B, w.gamma), dtype=torch.uint8, device=dev)
+    samp_ms = timed(lambda: gb.spec_sample_accept(s_draft, s_q, s_logits, s_u, s_n, s_t, ws_s))
+    # logits once, one draft row for the residual draw, the draft tokens' probabilities
+    samp_bytes = B * (w.gamma + 1) * w.vocab * 4 + B * w.vocab * 4 + B * w.gamma * 8 + B * (w.gamma + 1) * 4 + 8 * B
     del flush
     return {
+        "spec_sample_accept": {"avg_us": 1e3 * samp_ms, "algo_bytes_per_launch": samp_bytes,
+                               "achieved_gbs": samp_bytes / (samp_ms * 1e-3) / 1e9,
+                               "frac_of_peak": samp_bytes / (samp_ms * 1e-3) / 1e9 / peak,
+                               "accepted": [int(x) for x in s_n.cpu().tolist()],
+                               "shape": f"B={B} gamma={w.gamma} V={w.vocab} fp32 chain"},
         "cape_expand": {"avg_us": 1e3 * cape_ms, "algo_bytes_per_launch": cape_bytes,
                         "achieved_gbs": cape_bytes / (cape_ms * 1e-3) / 1e9,
                         "frac_of_peak": cape_bytes / (cape_ms * 1e-3) / 1e9 / peak,

@@ -25,6 +25,9 @@
  *                      tree_verify_attn and tree_accept take.
  *   glide_kv_compact   the cache update after acceptance (Section 3.1): the
  *                      accepted path's keys/values become contiguous rows.
+ *   spec_sample_accept speculative-sampling acceptance of a chain proposal
+ *                      (Section 2's other acceptance strategy, used for GliDe
+ *                      alone in Section 4.1), with caller-supplied uniforms.
  *
  * Conventions shared by all calls
  * -------------------------------
@@ -228,6 +231,35 @@ glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int
                               void* K_cache, void* V_cache, const int32_t* kv_len, int32_t n,
                               const int32_t* path, const int32_t* len, int32_t* new_kv_len,
                               glide_stream_t stream);
+
+/* Bytes of workspace that spec_sample_accept needs for B proposals of gamma tokens. */
+size_t glide_sample_workspace_bytes(int32_t B, int32_t gamma);
+
+/*
+ * Speculative-sampling acceptance of a chain proposal (the speculative
+ * sampling named in Section 2 and used for GliDe alone in Section 4.1; its
+ * outputs are distributed as the target model's own samples):
+ *   p_T,i = SoftMax(target_logits[b,i,:]) for i = 0..gamma (temperature 1);
+ *   position i (0-based) accepts draft_tokens[b,i] = x when
+ *     uniforms[b,i] * draft_probs[b,i,x] < p_T,i(x);
+ *   n_accepted[b] = the number of positions before the first rejection (gamma
+ *   if none);
+ *   next_token[b] = a draw from max(0, p_T,n - draft_probs[b,n,:]) if n < gamma,
+ *   else from p_T,gamma: the first token whose running weight exceeds
+ *   uniforms[b,gamma] * (total weight).  (If the residual weight sums to 0 in
+ *   fp32 the draw is from p_T,n.)
+ * The accepted tokens are draft_tokens[b,0..n-1], followed by next_token[b].
+ * The kernel computes in fp32; a result can differ from exact arithmetic only
+ * where a product u * p_D(x) or v * total lies within rounding of its threshold.
+ * draft_tokens [B,gamma] int32 (clamped to [0,V)), draft_probs [B,gamma,V] fp32,
+ * target_logits [B,gamma+1,V] fp32 finite and 16-byte aligned, uniforms
+ * [B,gamma+1] fp32 in [0,1), all on the device.  1 <= gamma <= 63, 1 <= V.
+ * Outputs n_accepted [B], next_token [B] int32.
+ */
+glide_status spec_sample_accept(const int32_t* draft_tokens, const float* draft_probs,
+                                const float* target_logits, const float* uniforms, int32_t B,
+                                int32_t gamma, int32_t V, int32_t* n_accepted, int32_t* next_token,
+                                void* workspace, size_t workspace_bytes, glide_stream_t stream);
 
 /*
  * glide_cross_attn for callers that cannot allocate device memory when they

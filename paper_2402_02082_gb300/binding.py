@@ -61,6 +61,9 @@ _SIG = {
                                    ctypes.c_int32, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "glide_kv_compact": (ctypes.c_int, [ctypes.POINTER(AttnDesc), ctypes.c_int32, ctypes.c_int64, _P, _P, _P,
                                         ctypes.c_int32, _P, _P, _P, _P]),
+    "glide_sample_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
+    "spec_sample_accept": (ctypes.c_int, [_P, _P, _P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _P, _P,
+                                          _P, ctypes.c_size_t, _P]),
 }
 
 
@@ -257,6 +260,30 @@ def glide_kv_compact(K_cache: torch.Tensor, V_cache: torch.Tensor, kv_len: torch
                                 new_kv_len.data_ptr(), _stream(stream))
     _check(st, "glide_kv_compact")
     return new_kv_len
+
+
+def glide_sample_workspace_bytes(B: int, gamma: int) -> int:
+    return int(lib().glide_sample_workspace_bytes(B, gamma))
+
+
+def spec_sample_accept(draft_tokens: torch.Tensor, draft_probs: torch.Tensor, target_logits: torch.Tensor,
+                       uniforms: torch.Tensor, n_accepted: torch.Tensor, next_token: torch.Tensor,
+                       workspace: torch.Tensor, stream=None):
+    """(n_accepted [B], next_token [B]) int32 <- speculative-sampling acceptance of the
+    chain draft_tokens [B, gamma] (draft_probs [B, gamma, V], target_logits [B, gamma+1, V],
+    uniforms [B, gamma+1])."""
+    B, gamma = draft_tokens.shape
+    V = target_logits.shape[-1]
+    for t, shp, dt in ((draft_tokens, (B, gamma), torch.int32), (draft_probs, (B, gamma, V), torch.float32),
+                       (target_logits, (B, gamma + 1, V), torch.float32), (uniforms, (B, gamma + 1), torch.float32),
+                       (n_accepted, (B,), torch.int32), (next_token, (B,), torch.int32)):
+        if t.dtype != dt or tuple(t.shape) != shp or not t.is_contiguous():
+            raise TypeError("spec_sample_accept: tensor of wrong dtype, shape or layout")
+    st = lib().spec_sample_accept(draft_tokens.data_ptr(), draft_probs.data_ptr(), target_logits.data_ptr(),
+                                  uniforms.data_ptr(), B, gamma, V, n_accepted.data_ptr(), next_token.data_ptr(),
+                                  workspace.data_ptr(), workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(st, "spec_sample_accept")
+    return n_accepted, next_token
 
 
 def glide_validate_tree(parent_idx_host, require_root0: bool = True) -> int:

@@ -199,6 +199,30 @@ glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int
   return from_cuda(glide::launch_kv_compact(a, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+size_t glide_sample_workspace_bytes(int32_t B, int32_t gamma) {
+  if (B < 1 || gamma < 1 || gamma > glide::kMaxTree - 1) return 0;
+  return glide::sample_workspace_bytes(B, gamma);
+}
+
+glide_status spec_sample_accept(const int32_t* draft_tokens, const float* draft_probs, const float* target_logits,
+                                const float* uniforms, int32_t B, int32_t gamma, int32_t V, int32_t* n_accepted,
+                                int32_t* next_token, void* workspace, size_t workspace_bytes,
+                                glide_stream_t stream) {
+  if (B < 1 || gamma < 1 || gamma > glide::kMaxTree - 1 || V < 1) return GLIDE_ERR_INVALID;
+  if ((double)B * (gamma + 1) * V > 4.0e18) return GLIDE_ERR_INVALID;
+  if (!draft_tokens || !draft_probs || !target_logits || !uniforms || !n_accepted || !next_token || !workspace)
+    return GLIDE_ERR_INVALID;
+  if (!aligned16(target_logits) || !aligned16(workspace) || (reinterpret_cast<uintptr_t>(draft_probs) & 3u) ||
+      (reinterpret_cast<uintptr_t>(draft_tokens) & 3u) || (reinterpret_cast<uintptr_t>(uniforms) & 3u) ||
+      (reinterpret_cast<uintptr_t>(n_accepted) & 3u) || (reinterpret_cast<uintptr_t>(next_token) & 3u))
+    return GLIDE_ERR_INVALID;
+  if (workspace_bytes < glide::sample_workspace_bytes(B, gamma)) return GLIDE_ERR_INVALID;
+  glide::SampleArgs a;
+  a.draft = draft_tokens; a.q = draft_probs; a.logits = target_logits; a.u = uniforms;
+  a.B = B; a.gamma = gamma; a.V = V; a.n_acc = n_accepted; a.next_tok = next_token; a.ws = workspace;
+  return from_cuda(glide::launch_spec_sample(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 glide_status glide_validate_tree(const int32_t* parent_idx_host, int32_t B, int32_t n, int32_t require_root0) {
   if (!parent_idx_host || B < 1 || n < 1) return GLIDE_ERR_INVALID;
   for (int32_t b = 0; b < B; ++b) {

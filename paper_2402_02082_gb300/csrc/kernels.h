@@ -66,6 +66,17 @@ struct CompactArgs {
   int dtype;               // 0 bf16, 1 f32
 };
 
+struct SampleArgs {
+  const int32_t* draft;   // [B, gamma]
+  const float* q;         // [B, gamma, V]
+  const float* logits;    // [B, gamma + 1, V]
+  const float* u;         // [B, gamma + 1]
+  int B, gamma, V;
+  int32_t* n_acc;         // [B]
+  int32_t* next_tok;      // [B]
+  void* ws;
+};
+
 int sm_count();  // multiprocessors of the current device (cached per device)
 
 cudaError_t launch_cross_attn(const AttnArgs& a, cudaStream_t st);
@@ -76,8 +87,10 @@ cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st);
 
 cudaError_t launch_cape_expand(const CapeArgs& a, cudaStream_t st);
 cudaError_t launch_kv_compact(const CompactArgs& a, cudaStream_t st);
+cudaError_t launch_spec_sample(const SampleArgs& a, cudaStream_t st);
 
 size_t accept_workspace_bytes(int B, int n);
 size_t cape_workspace_bytes(int B, int gamma, int V);
+size_t sample_workspace_bytes(int B, int gamma);
 
 }  // namespace glide

@@ -180,6 +180,34 @@ def root_tokens(seed: int, B: int, vocab: int) -> np.ndarray:
     return _rng(seed, 32).integers(vocab, size=B).astype(np.int32)
 
 
+def sample_tokens(seed: int, probs: np.ndarray) -> np.ndarray:
+    """One token drawn from each distribution of probs [..., V] (the draft
+    model's own sampling of its proposal)."""
+    g = _rng(seed, 33)
+    flat = probs.reshape(-1, probs.shape[-1]).astype(np.float64)
+    out = np.array([g.choice(flat.shape[1], p=row / row.sum()) for row in flat], dtype=np.int32)
+    return out.reshape(probs.shape[:-1])
+
+
+def target_logits_near(seed: int, draft_probs: np.ndarray, mix: float, extra_rows: int = 1) -> np.ndarray:
+    """fp32 target logits [B, gamma + extra_rows, V] whose distributions mix the
+    draft's (weight `mix`) with independent heavy-tailed ones, so that a
+    proposal is accepted part of the time; the extra rows are independent."""
+    g = _rng(seed, 34)
+    B, gamma, V = draft_probs.shape
+    other = g.gamma(0.3, size=(B, gamma + extra_rows, V))
+    other /= other.sum(-1, keepdims=True)
+    p = other.copy()
+    p[:, :gamma] = mix * draft_probs.astype(np.float64) + (1.0 - mix) * other[:, :gamma]
+    return np.log(np.maximum(p, 1e-30)).astype(np.float32)
+
+
+def uniforms(seed: int, shape) -> np.ndarray:
+    """fp32 uniform numbers in [0, 1) (the random numbers a sampling step draws)."""
+    u = _rng(seed, 35).random(size=tuple(shape)).astype(np.float32)
+    return np.minimum(u, np.float32(0.99999994))
+
+
 # --------------------------------------------------------------------------
 # workloads
 # --------------------------------------------------------------------------

@@ -143,3 +143,16 @@ def test_binding_refuses_missing_library(monkeypatch, tmp_path):
     monkeypatch.setattr(gb, "library_path", lambda: str(tmp_path / "absent.so"))
     with pytest.raises(RuntimeError, match="not found"):
         gb.lib()
+
+
+def test_spec_sample_rejects(L):
+    assert gb.glide_sample_workspace_bytes(4, 5) > 0
+    assert gb.glide_sample_workspace_bytes(0, 5) == 0 and gb.glide_sample_workspace_bytes(4, 0) == 0
+    assert gb.glide_sample_workspace_bytes(4, 64) == 0
+
+    def ss(d=FAKE, q=FAKE, lg=FAKE, u=FAKE, B=2, g=5, V=100, n=FAKE, t=FAKE, ws=FAKE, wsb=1 << 20):
+        return L.spec_sample_accept(d, q, lg, u, B, g, V, n, t, ws, wsb, None)
+    for b in [dict(B=0), dict(g=0), dict(g=64), dict(V=0), dict(d=None), dict(q=None), dict(lg=None), dict(u=None),
+              dict(n=None), dict(t=None), dict(ws=None), dict(wsb=16), dict(lg=FAKE + 4), dict(q=FAKE + 2),
+              dict(ws=FAKE + 8)]:
+        assert ss(**b) == gb.GLIDE_ERR_INVALID, b
