@@ -5,7 +5,7 @@ values K^{l,j}, V^{l,j} (Section 3.1); the draft query Q^{m,j}; scale
 1/sqrt(d_k).  Tensor layouts are those of the library boundary:
 
     queries  [B, nq, H, D]
-    K, V     [B, H, S_cap, D]   (rows >= kv_len[b] + n are unused capacity)
+    K, V     [B, H_kv, S_cap, D] (rows >= kv_len[b] + n are unused capacity)
     kv_len   [B]
     parent   [B, n]  (-1 for a root, else an earlier node)
 
@@ -47,6 +47,16 @@ def _softmax_rows_attend(scores: np.ndarray, allowed: np.ndarray, values: np.nda
     return out
 
 
+def kv_head(h: int, H: int, H_kv: int) -> int:
+    """The cached key/value head that query head h reads.  H_kv = H is plain
+    multi-head attention; with fewer cached heads (grouped-query attention, as
+    in Mistral-7B: 32 query heads over 8 key/value heads) each run of H / H_kv
+    consecutive query heads shares one cached head."""
+    if H % H_kv:
+        raise ValueError("the query heads must split evenly over the key/value heads")
+    return h // (H // H_kv)
+
+
 def _pairs(B: int, H: int, pairs: Optional[Iterable[Tuple[int, int]]]):
     if pairs is None:
         return [(b, h) for b in range(B) for h in range(H)]
@@ -69,8 +79,9 @@ def cross_attn(q_draft: np.ndarray, K: np.ndarray, V: np.ndarray, kv_len: Sequen
     out = np.full((B, nq, H, D), np.nan)
     for b, h in _pairs(B, H, pairs):
         L = int(kv_len[b])
-        Kb = widen(K[b, h, :L])
-        Vb = widen(V[b, h, :L])
+        hk = kv_head(h, H, K.shape[1])
+        Kb = widen(K[b, hk, :L])
+        Vb = widen(V[b, hk, :L])
         Q = widen(q_draft[b, :, h, :])                  # [nq, D]
         scores = (Q @ Kb.T) * sc                        # Q K^T / sqrt(d_k)
         allowed = np.ones_like(scores, dtype=bool)
@@ -124,8 +135,9 @@ def tree_verify_attn(q_tree: np.ndarray, parent_idx: np.ndarray, K: np.ndarray, 
         L = int(kv_len[b])
         if b not in masks:
             masks[b] = tree_allowed_mask(parent_idx[b], L)
-        Kb = widen(K[b, h, :L + n])
-        Vb = widen(V[b, h, :L + n])
+        hk = kv_head(h, H, K.shape[1])
+        Kb = widen(K[b, hk, :L + n])
+        Vb = widen(V[b, hk, :L + n])
         Q = widen(q_tree[b, :, h, :])
         scores = (Q @ Kb.T) * sc
         out[b, :, h, :] = _softmax_rows_attend(scores, masks[b], Vb)

@@ -690,3 +690,32 @@ def check_spec_sample_same_model_accepts(spec_sample_accept):
         p = np.exp(z[b, gamma] - z[b, gamma].max())
         c = np.cumsum(p / p.sum())
         assert int(tok[b]) == int(np.searchsorted(c, float(u[b, gamma]), side="right"))
+
+
+# ------------------------------------------------ grouped-query attention
+def check_gqa_is_repeated_kv(cross_attn, tree_verify_attn):
+    """Grouped-query attention (the cached heads fewer than the query heads, as
+    in Mistral-7B) is multi-head attention over cached heads repeated so that
+    each run of H / H_kv consecutive query heads sees its own copy."""
+    g = _rng(40)
+    for H, H_kv in ((8, 2), (6, 3), (4, 1), (4, 4)):
+        B, D, n = 2, 16, 5
+        L = [9, 4]
+        S = max(L) + n
+        K = g.standard_normal((B, H_kv, S, D)).astype(np.float32)
+        V = g.standard_normal((B, H_kv, S, D)).astype(np.float32)
+        Kr, Vr = np.repeat(K, H // H_kv, axis=1), np.repeat(V, H // H_kv, axis=1)
+        qd = g.standard_normal((B, 1, H, D)).astype(np.float32)
+        assert np.allclose(cross_attn(qd, K, V, L), cross_attn(qd, Kr, Vr, L), rtol=1e-12, atol=1e-12), (H, H_kv)
+        qt = g.standard_normal((B, n, H, D)).astype(np.float32)
+        parent = np.stack([random_small_tree(g, n) for _ in range(B)])
+        assert np.allclose(tree_verify_attn(qt, parent, K, V, L), tree_verify_attn(qt, parent, Kr, Vr, L),
+                           rtol=1e-12, atol=1e-12), (H, H_kv)
+        # and a query head reads exactly its group's cached head: changing another
+        # group's cache leaves it alone
+        if H_kv > 1:
+            K2 = K.copy()
+            K2[:, 1:] += g.standard_normal(K2[:, 1:].shape).astype(np.float32)
+            o1, o2 = cross_attn(qd, K, V, L), cross_attn(qd, K2, V, L)
+            grp = H // H_kv
+            assert np.allclose(o1[:, :, :grp], o2[:, :, :grp]) and not np.allclose(o1[:, :, grp:], o2[:, :, grp:])

@@ -387,3 +387,14 @@ def test_mutant_sampling_bonus_from_last_proposal_row():
         return n, np.where(n == gamma, tok2, tok)
     _expect_some_fail([lambda: pins.check_spec_sample_golden(bad),
                        lambda: pins.check_spec_sample_same_model_accepts(bad)])
+
+
+# ------------------------------------------------ grouped-query attention
+def test_gqa_is_repeated_kv():
+    pins.check_gqa_is_repeated_kv(oracle.cross_attn, oracle.tree_verify_attn)
+
+
+def test_mutant_gqa_interleaved_heads(monkeypatch):
+    # query head h reading cached head h % H_kv (interleaved) instead of its group's
+    monkeypatch.setattr(oatt, "kv_head", lambda h, H, H_kv: h % H_kv)
+    _expect_some_fail([lambda: pins.check_gqa_is_repeated_kv(oracle.cross_attn, oracle.tree_verify_attn)])
