@@ -37,7 +37,10 @@
  *   asynchronous: a returned GLIDE_OK means "launched", not "finished".
  * - Layouts are dense, row-major, no padding:
  *     queries   [B, nq, H, D]          (nq = 1 for cross-attention, n for the tree)
- *     K, V      [B, H, S_cap, D]       one contiguous S_cap x D slab per (b, h)
+ *     K, V      [B, H_kv, S_cap, D]    one contiguous S_cap x D slab per (b, cached
+ *                                      head); H_kv = H is multi-head attention, fewer
+ *                                      cached heads is grouped-query attention: query
+ *                                      head h reads cached head h / (H / H_kv)
  *     out       [B, nq, H, D] fp32
  *     kv_len    [B] int32              cached prefix length of each sequence
  *     parent    [B, n] int32           linearized tree: -1 for a root, else an
@@ -73,7 +76,7 @@
 extern "C" {
 #endif
 
-#define GLIDE_ABI_VERSION 1
+#define GLIDE_ABI_VERSION 2
 
 typedef struct CUstream_st* glide_stream_t;
 
@@ -93,13 +96,17 @@ typedef enum { GLIDE_BF16 = 0, GLIDE_F32 = 1 } glide_dtype;
 
 typedef struct {
   int32_t B;          /* sequences in the batch, 1..1024                                   */
-  int32_t H;          /* attention heads (of the target layer), >= 1                       */
+  int32_t H;          /* query heads (of the target layer), >= 1                            */
   int32_t D;          /* head dimension d_k: 64 or 128                                     */
   int32_t S_cap;      /* rows of each (b, h) slab of the K/V cache                          */
   glide_dtype dtype;  /* element type of queries, K and V                                   */
   float scale;        /* softmax scale; 0 means 1/sqrt(D) (Section 3.1)                     */
   uint32_t flags;     /* GLIDE_FLAG_* bits                                                  */
   int32_t max_ctas;   /* upper bound on the CTAs of one attention launch; 0 = automatic     */
+  int32_t H_kv;       /* cached (key/value) heads; 0 means H.  H % H_kv == 0: each run of
+                         H / H_kv consecutive query heads shares one cached head (grouped-
+                         query attention, as in Mistral-7B: 32 query over 8 cached heads).
+                         tree_verify_attn needs n * H / H_kv <= 64.                       */
 } glide_attn_desc;
 
 /* Version of this ABI (GLIDE_ABI_VERSION of the built library). */

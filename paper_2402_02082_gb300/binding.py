@@ -37,7 +37,7 @@ class GlideError(RuntimeError):
 class AttnDesc(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("D", ctypes.c_int32),
                 ("S_cap", ctypes.c_int32), ("dtype", ctypes.c_int), ("scale", ctypes.c_float),
-                ("flags", ctypes.c_uint32), ("max_ctas", ctypes.c_int32)]
+                ("flags", ctypes.c_uint32), ("max_ctas", ctypes.c_int32), ("H_kv", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -118,8 +118,9 @@ def _dtype_code(t: torch.Tensor) -> int:
 
 
 def make_desc(B: int, H: int, D: int, S_cap: int, dtype: int, scale: float = 0.0, flags: int = 0,
-              max_ctas: int = 0) -> AttnDesc:
-    return AttnDesc(B, H, D, S_cap, dtype, scale, flags, max_ctas)
+              max_ctas: int = 0, H_kv: int = 0) -> AttnDesc:
+    """H query heads; H_kv cached heads (0: H; fewer: grouped-query attention)."""
+    return AttnDesc(B, H, D, S_cap, dtype, scale, flags, max_ctas, H_kv)
 
 
 def glide_attn_workspace_bytes(desc: AttnDesc, n_queries: int) -> int:
@@ -131,13 +132,15 @@ def glide_accept_workspace_bytes(B: int, n: int) -> int:
 
 
 def _cache_desc(q: torch.Tensor, K: torch.Tensor, V: torch.Tensor, scale, flags, max_ctas) -> AttnDesc:
-    if K.dim() != 4 or V.shape != K.shape or K.dtype != V.dtype or q.dtype != K.dtype:
-        raise ValueError("K/V must be [B, H, S_cap, D] of the queries' dtype")
+    """Descriptor from queries [B, nq, H, D] and caches [B, H_kv, S_cap, D]."""
+    if K.dim() != 4 or V.shape != K.shape or K.dtype != V.dtype or q.dtype != K.dtype or q.dim() != 4:
+        raise ValueError("K/V must be [B, H_kv, S_cap, D] of the queries' dtype")
     for t in (q, K, V):
         if not t.is_contiguous():
             raise ValueError("tensors must be contiguous")
-    B, H, S_cap, D = K.shape
-    return make_desc(B, H, D, S_cap, _dtype_code(K), scale, flags, max_ctas)
+    B, H_kv, S_cap, D = K.shape
+    H = q.shape[2]
+    return make_desc(B, H, D, S_cap, _dtype_code(K), scale, flags, max_ctas, H_kv=H_kv if H_kv != H else 0)
 
 
 def glide_cross_attn(q_draft: torch.Tensor, K_cache: torch.Tensor, V_cache: torch.Tensor, kv_len: torch.Tensor,

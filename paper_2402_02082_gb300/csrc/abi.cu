@@ -31,17 +31,21 @@ namespace {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Cached (key/value) heads: H_kv, or H when it is 0.
+int hkv(const glide_attn_desc* d) { return d->H_kv > 0 ? d->H_kv : d->H; }
+
 bool desc_ok(const glide_attn_desc* d) {
   if (!d) return false;
   if (d->B < 1 || d->B > glide::kMaxBatch) return false;
   if (d->H < 1 || d->H > 65535) return false;
+  if (d->H_kv < 0 || d->H_kv > d->H || d->H % hkv(d) != 0) return false;
   if (d->D != 64 && d->D != 128) return false;
   if (d->S_cap < 1) return false;
   if (d->dtype != GLIDE_BF16 && d->dtype != GLIDE_F32) return false;
   if (!(d->scale >= 0.f) || isinf(d->scale)) return false;  // rejects NaN and negatives
   if (d->max_ctas < 0) return false;
   // every element offset must fit comfortably in 63 bits
-  const double elems = (double)d->B * d->H * (double)d->S_cap * d->D;
+  const double elems = (double)d->B * d->H * (double)d->S_cap * d->D;  // >= the cache (H_kv <= H)
   if (elems > 4.0e18) return false;
   return true;
 }
@@ -49,8 +53,11 @@ bool desc_ok(const glide_attn_desc* d) {
 size_t attn_ws_bytes(const glide_attn_desc* d, int nq) {
   // partial slots: one per (share or chunk, b, h) pair index; a tree slot holds
   // nq query rows, a cross-attention slot one row per consumer warp
-  const size_t slots = (size_t)glide::kMaxCtas + (size_t)d->B * d->H;
-  const size_t rows = (size_t)(nq > glide::kCrossPartials ? nq : glide::kCrossPartials);
+  // (with grouped-query attention a slab is a (b, cached head) and holds
+  // nq x group query rows)
+  const size_t slots = (size_t)glide::kMaxCtas + (size_t)d->B * hkv(d);
+  const size_t q_rows = (size_t)nq * (d->H / hkv(d));
+  const size_t rows = q_rows > (size_t)glide::kCrossPartials ? q_rows : (size_t)glide::kCrossPartials;
   return glide::WsLayout::partials_off(d->B, d->H) + slots * rows * (d->D + 2) * sizeof(float);
 }
 
@@ -60,6 +67,8 @@ glide::AttnArgs make_args(const glide_attn_desc* d, const void* q, const void* K
   glide::AttnArgs a;
   a.q = q; a.K = K; a.V = V; a.kv_len = kv_len; a.parent = parent; a.out = out; a.ws = ws;
   a.B = d->B; a.H = d->H; a.D = d->D; a.S_cap = d->S_cap; a.nq = nq; a.max_kv_len = max_kv_len;
+  a.Hkv = hkv(d);
+  a.tree = parent != nullptr ? 1 : 0;
   a.dtype = d->dtype == GLIDE_BF16 ? 0 : 1;
   a.scale = d->scale > 0.f ? d->scale : 1.0f / sqrtf((float)d->D);
   a.flags = d->flags;
@@ -88,6 +97,7 @@ const char* glide_status_str(glide_status s) {
 
 size_t glide_attn_workspace_bytes(const glide_attn_desc* desc, int32_t n_queries) {
   if (!desc_ok(desc) || n_queries < 1 || n_queries > glide::kMaxTree) return 0;
+  if (n_queries * (desc->H / hkv(desc)) > glide::kMaxTree) return 0;
   return attn_ws_bytes(desc, n_queries);
 }
 
@@ -112,7 +122,17 @@ glide_status glide_cross_attn(const glide_attn_desc* desc, const void* q_draft, 
   if (max_kv_len < 1 || max_kv_len > desc->S_cap) return GLIDE_ERR_INVALID;
   if (workspace_bytes < attn_ws_bytes(desc, 1)) return GLIDE_ERR_INVALID;
   glide::AttnArgs a = make_args(desc, q_draft, K_cache, V_cache, kv_len, nullptr, out, workspace, 1, max_kv_len);
-  return from_cuda(glide::launch_cross_attn(a, reinterpret_cast<cudaStream_t>(stream)));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (a.Hkv == a.H) return from_cuda(glide::launch_cross_attn(a, st));
+  // Grouped-query attention: a cached head serves H / H_kv draft queries, so
+  // one pass over its keys is a small dense contraction -- the verification
+  // kernels without tree keys, with the group's queries as their rows.
+  if (a.H / a.Hkv > glide::kMaxTree) return GLIDE_ERR_UNSUPPORTED;
+  if (!(a.flags & GLIDE_FLAG_FORCE_FMA)) {
+    cudaError_t e = glide::launch_tree_attn_tc(a, st);
+    if (e != cudaErrorNotSupported) return from_cuda(e);
+  }
+  return from_cuda(glide::launch_tree_attn_fma(a, st));
 }
 
 glide_status tree_verify_attn(const glide_attn_desc* desc, const void* q_tree, int32_t n, const int32_t* parent_idx,
@@ -126,6 +146,7 @@ glide_status tree_verify_attn(const glide_attn_desc* desc, const void* q_tree, i
       (reinterpret_cast<uintptr_t>(parent_idx) & 3u))
     return GLIDE_ERR_INVALID;
   if (max_kv_len < 0 || (long long)max_kv_len + n > desc->S_cap) return GLIDE_ERR_INVALID;
+  if (n * (desc->H / hkv(desc)) > glide::kMaxTree) return GLIDE_ERR_UNSUPPORTED;  // query rows of a slab
   if (workspace_bytes < attn_ws_bytes(desc, n)) return GLIDE_ERR_INVALID;
   glide::AttnArgs a = make_args(desc, q_tree, K_cache, V_cache, kv_len, parent_idx, out, workspace, n, max_kv_len);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -180,7 +201,7 @@ glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int
   if (!desc_ok(desc)) return GLIDE_ERR_INVALID;
   if (n < 1 || n > glide::kMaxTree || n > desc->S_cap) return GLIDE_ERR_INVALID;
   if (n_layers < 1) return GLIDE_ERR_INVALID;
-  const int64_t layer_elems = (int64_t)desc->B * desc->H * desc->S_cap * desc->D;
+  const int64_t layer_elems = (int64_t)desc->B * hkv(desc) * desc->S_cap * desc->D;  // the cache's heads
   if (n_layers > 1 && layer_stride < layer_elems) return GLIDE_ERR_INVALID;
   if ((double)n_layers * (double)(n_layers > 1 ? layer_stride : layer_elems) > 4.0e18) return GLIDE_ERR_INVALID;
   const int elt = desc->dtype == GLIDE_BF16 ? 2 : 4;
@@ -194,7 +215,7 @@ glide_status glide_kv_compact(const glide_attn_desc* desc, int32_t n_layers, int
   glide::CompactArgs a;
   a.K = K_cache; a.V = V_cache; a.kv_len = kv_len; a.path = path; a.len = len; a.new_kv_len = new_kv_len;
   a.layers = n_layers; a.layer_stride = n_layers > 1 ? layer_stride : layer_elems;
-  a.B = desc->B; a.H = desc->H; a.D = desc->D; a.S_cap = desc->S_cap; a.n = n;
+  a.B = desc->B; a.H = hkv(desc); a.D = desc->D; a.S_cap = desc->S_cap; a.n = n;
   a.dtype = desc->dtype == GLIDE_BF16 ? 0 : 1;
   return from_cuda(glide::launch_kv_compact(a, reinterpret_cast<cudaStream_t>(stream)));
 }

@@ -185,12 +185,21 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Output row of query row r of slab (b, cached head h): rows are node-major,
+// `group` query heads per node, Hq query heads in all (group = 1, Hq = H: one
+// query head per slab).
+__device__ __forceinline__ size_t out_row(int b, int h, int r, int nrows, int group, int Hq) {
+  const int node = r / group;
+  return ((size_t)b * (nrows / group) + node) * Hq + (size_t)h * group + (r - node * group);
+}
+
 // After this CTA wrote its partial for (b, h) into its slot, count the CTA in;
 // the CTA that completes the count merges every slot of (b, h) into `out` and
-// re-arms the counter.  Nothing waits: the last arrival does the work.
+// re-arms the counter.  Nothing waits: the last arrival does the work.  (b, h)
+// is a slab of cached head h; its nq query rows map to outputs by out_row.
 // Called by all `nthreads` consumer threads.
-__device__ inline void combine_if_last(const Segment& s, int B, int H, int nq, int D, float* partials,
-                                       unsigned* counters, float* out, int ctid, int nthreads,
+__device__ inline void combine_if_last(const Segment& s, int B, int H, int nq, int D, int group, int Hq,
+                                       float* partials, unsigned* counters, float* out, int ctid, int nthreads,
                                        volatile int* flag) {
   const int bh = s.b * H + s.h;
   __threadfence();
@@ -216,7 +225,7 @@ __device__ inline void combine_if_last(const Segment& s, int B, int H, int nq, i
         L += w * __ldcg(row + 1);
         O += w * __ldcg(row + 2 + d);
       }
-      out[(((size_t)s.b * nq + iq) * H + s.h) * D + d] = O / L;
+      out[out_row(s.b, s.h, iq, nq, group, Hq) * D + d] = O / L;
     }
     if (ctid == 0) counters[bh] = 0u;
   }
@@ -239,7 +248,8 @@ __device__ inline bool arrive_split(const Segment& s, int H, unsigned* counters,
   return *flag != 0;
 }
 
-// Merges every split partial of (b, h) = (s.b, s.h) into `out` and re-arms
+// Merges every split partial of slab (b, h) = (s.b, s.h) into `out` (query
+// rows placed by out_row) and re-arms
 // the counter; all `nthreads` threads of the CTA call it (it uses
 // __syncthreads).  scratch: shared memory for (2 + kCombineW) * nq floats.
 // Pass 1, one thread per query row: M = max_c m_c, the weights
@@ -247,8 +257,9 @@ __device__ inline bool arrive_split(const Segment& s, int H, unsigned* counters,
 // thread taking kCombineU of them with every load issued before any use.
 constexpr int kCombineW = 8;   // slots whose weights are kept in shared memory
 constexpr int kCombineU = 3;   // outputs per thread per round
-__device__ inline void combine_partials(const Segment& s, int H, int nq, int D, const float* partials,
-                                        unsigned* counters, float* out, float* scratch, int tid, int nthreads) {
+__device__ inline void combine_partials(const Segment& s, int H, int nq, int D, int group, int Hq,
+                                        const float* partials, unsigned* counters, float* out, float* scratch,
+                                        int tid, int nthreads) {
   const int bh = s.b * H + s.h;
   const int nsl = s.c_last - s.c_first + 1;
   const int rs = D + 2;  // floats per partial row: m, l, o[D]
@@ -338,7 +349,7 @@ __device__ inline void combine_partials(const Segment& s, int H, int nq, int D, 
       if (it < items) {
         const int r = it / cpr, d0 = (it - r * cpr) * 4;
         const float li = Linv[r];
-        *reinterpret_cast<float4*>(out + (((size_t)s.b * nq + r) * H + s.h) * D + d0) =
+        *reinterpret_cast<float4*>(out + out_row(s.b, s.h, r, nq, group, Hq) * D + d0) =
             make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
       }
     }

@@ -22,6 +22,8 @@ struct AttnArgs {
   void* ws;
   int B, H, D, S_cap;
   int nq;                 // queries per (b, h): 1 for cross-attention, n for the tree
+  int Hkv;                // cached (key/value) heads; H % Hkv == 0, H / Hkv query heads per cached head
+  int tree;               // 1: the nq tree keys follow the prefix (verification); 0: prefix only
   int max_kv_len;
   int dtype;              // 0 bf16, 1 f32
   float scale;            // already resolved (never 0)

@@ -1,6 +1,9 @@
-// Tree verification attention on CUDA cores (Section 3.2): n <= 64 tree
-// queries per (sequence, head) attend to every cached prefix key and to the
-// tree keys of their ancestors and themselves.  The CaPE mask is this
+// Tree verification attention on CUDA cores (Section 3.2): n tree queries per
+// (sequence, head) attend to every cached prefix key and to the tree keys of
+// their ancestors and themselves.  With grouped-query attention a slab is a
+// (sequence, cached head) and serves the n x group query rows of the heads
+// that share it (at most 64); without tree keys (prefix only) the same kernel
+// is grouped-query cross-attention.  The CaPE mask is this
 // ancestor-or-self mask on CaPE's trees (proposal spine plus expansion
 // leaves); the kernel takes any parent array.
 //
@@ -50,6 +53,10 @@ struct TreeParams {
   unsigned* counters;
   float* partials;
   int B, H, S_cap, max_kv_len, n;
+  int Hkv;    // cached heads (slabs are (b, cached head))
+  int group;  // query heads per cached head (H / Hkv)
+  int rows;   // query rows per slab: n nodes x group heads, node-major, <= 64
+  int tree;   // 1: the n tree keys follow the prefix (verification); 0: prefix only
   float scale_log2;
 };
 
@@ -82,7 +89,13 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
     *abort_flag = 0;
     fence_barrier_init();
   }
-  build_batch_tiles(bt, p.kv_len, p.B, p.H, p.max_kv_len, n, kTK);
+  build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);
+  if (!p.tree) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
+    const long long total = (long long)p.B * n * p.H * D;
+    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x)
+      if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
+  }
 
   Partition P;
   P.init(bt.start[p.B], gridDim.x);
@@ -97,7 +110,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       bool ok = true;
       for (long long g = g_begin; g < g_end && ok;) {
         const Segment s = locate(bt, P, p.B, g, g_end);
-        const size_t slab = ((size_t)s.b * p.H + s.h) * p.S_cap;
+        const size_t slab = ((size_t)s.b * p.Hkv + s.h) * p.S_cap;
         for (int t = s.t0; t < s.t1; ++t, ++i) {
           const int st = i % NS;
           if (!mbar_wait(&empty[st], ((i / NS) & 1) ^ 1, abort_flag, p.status)) { ok = false; break; }
@@ -128,7 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
     const int plen = bt.plen[s.b];
 
     // ancestor-or-self set of every node; a parent outside [-1, j) ends the walk
-    if (ctid < n) {
+    if (ctid < n && p.tree) {  // prefix only: no tree keys, no parent array
       uint64_t mask = 0;
       int j = ctid;
       for (int step = 0; step < kMaxTree && j >= 0; ++step) {
@@ -142,6 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
 
     float q[kQPW][E], o[kQPW][E], m[kQPW], l[kQPW];
     uint64_t am[kQPW];
+    // query row iq of the slab: node iq / group, head s.h * group + iq % group
 #pragma unroll
     for (int j = 0; j < kQPW; ++j) {
       const int iq = warp + j * kNW;
@@ -150,12 +164,13 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       am[j] = 0;
 #pragma unroll
       for (int e = 0; e < E; ++e) { o[j][e] = 0.f; q[j][e] = 0.f; }
-      if (iq < n) {
-        load_row_chunk<T, E>(static_cast<const T*>(p.q) + (((size_t)s.b * n + iq) * p.H + s.h) * D + lane * E,
+      if (iq < p.rows) {
+        const int node = iq / p.group;
+        load_row_chunk<T, E>(static_cast<const T*>(p.q) + out_row(s.b, s.h, iq, p.rows, p.group, p.H) * D + lane * E,
                              q[j]);
 #pragma unroll
         for (int e = 0; e < E; ++e) q[j][e] *= sl2;
-        am[j] = anc[iq];
+        am[j] = p.tree ? anc[node] : 0ull;
       }
     }
 
@@ -169,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       const T* Vt = sV + (size_t)st * kTK * D + lane * E;
 #pragma unroll
       for (int j = 0; j < kQPW; ++j) {
-        if (warp + j * kNW >= n) break;
+        if (warp + j * kNW >= p.rows) break;
         float part[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
@@ -207,16 +222,16 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       if (lane == 0) mbar_arrive(&empty[st]);
     }
 
-    const int bh = s.b * p.H + s.h;
+    const int bh = s.b * p.Hkv + s.h;
     const bool single = s.c_first == s.c_last;
-    float* slot = partial_slot(p.partials, blockIdx.x + bh, n, D);
+    float* slot = partial_slot(p.partials, blockIdx.x + bh, p.rows, D);
 #pragma unroll
     for (int j = 0; j < kQPW; ++j) {
       const int iq = warp + j * kNW;
-      if (iq >= n) break;
+      if (iq >= p.rows) break;
       const float L = warp_sum(l[j]);
       if (single) {
-        float* dst = p.out + (((size_t)s.b * n + iq) * p.H + s.h) * D + lane * E;
+        float* dst = p.out + out_row(s.b, s.h, iq, p.rows, p.group, p.H) * D + lane * E;
 #pragma unroll
         for (int e = 0; e < E; ++e) dst[e] = o[j][e] / L;
       } else {
@@ -227,7 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       }
     }
     if (single) consumer_sync(kCT);
-    else combine_if_last(s, p.B, p.H, n, D, p.partials, p.counters, p.out, ctid, kCT, last_flag);
+    else combine_if_last(s, p.B, p.Hkv, p.rows, D, p.group, p.H, p.partials, p.counters, p.out, ctid, kCT, last_flag);
     i_base += ntile;
     g = s.g_end;
   }
@@ -243,7 +258,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  const long long tiles_ub = (long long)a.B * a.H * ((a.max_kv_len + a.nq + kTK - 1) / kTK);
+  const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
   long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
@@ -255,6 +270,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
   p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
+  p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.rows = a.nq * p.group; p.tree = a.tree;
   p.scale_log2 = a.scale * kLog2e;
   tree_attn_fma_kernel<T, D><<<(unsigned)G, kThreads, C::smem_bytes(a.B), st>>>(p);
   return cudaGetLastError();
@@ -263,6 +279,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 }  // namespace
 
 cudaError_t launch_tree_attn_fma(const AttnArgs& a, cudaStream_t st) {
+  if (a.nq * (a.H / a.Hkv) > kMaxTree) return cudaErrorInvalidValue;  // the abi rejects this first
   if (a.dtype == 0 && a.D == 128) return launch_typed<__nv_bfloat16, 128>(a, st);
   if (a.dtype == 0 && a.D == 64) return launch_typed<__nv_bfloat16, 64>(a, st);
   if (a.dtype == 1 && a.D == 128) return launch_typed<float, 128>(a, st);

@@ -107,6 +107,10 @@ struct TcParams {
   unsigned* counters;
   float* partials;
   int B, H, S_cap, max_kv_len, n;
+  int Hkv;    // cached heads (slabs are (b, cached head))
+  int group;  // query heads per cached head (H / Hkv)
+  int rows;   // query rows per slab: n nodes x group heads, node-major, <= 64
+  int tree;   // 1: the n tree keys follow the prefix (verification); 0: prefix only
   int ns;  // K/V stages
   float scale_log2;
 };
@@ -179,7 +183,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
-  build_batch_tiles(bt, p.kv_len, p.B, p.H, p.max_kv_len, n, kTK);  // __syncthreads inside
+  build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);  // __syncthreads inside
+  if (!p.tree) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
+    const long long total = (long long)p.B * n * p.H * D;
+    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x)
+      if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
+  }
   tc::fence_after_sync();
   const uint32_t tmem = *tmem_slot;
 
@@ -210,7 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue = [&](Cursor& c, const CUtensorMap* map, uint64_t* full, uint32_t dst0) {
         const int st = c.i % ns;
         mbar_arrive_expect_tx(&full[st], C::kKVTile);
-        const int row = (c.s.b * p.H + c.s.h) * p.S_cap + c.t * kTK;
+        const int row = (c.s.b * p.Hkv + c.s.h) * p.S_cap + c.t * kTK;
         for (int hd = 0; hd < C::kHalves; ++hd)
           tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, row, &full[st], pol);
         ++c.i;
@@ -333,8 +343,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rr = (lane >> 2) + 8 * (lane & 1);  // row within the quarter
     const int cpar = (lane >> 1) & 1;             // column parity of this thread
     const int row = quarter * 16 + rr;            // MMA row
-    const int qi = rr * 4 + quarter;              // the tree query in this row
-    const bool valid = qi < n;
+    const int qi = rr * 4 + quarter;              // the query row of this MMA row
+    const bool valid = qi < p.rows;
+    const int node = valid ? qi / p.group : 0;    // its tree node (the draft query for cross-attention)
+    const int gi = valid ? qi - node * p.group : 0;  // its head within the slab's group
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t o_col = C::kTmemO + half * D;
     const int sid = threadIdx.x;                  // 0..255 among the softmax threads
@@ -347,7 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto write_q = [&](const Segment& sq, int sg) {
       unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
       const uint4* src =
-          reinterpret_cast<const uint4*>(p.q + (((size_t)sq.b * n + (valid ? qi : 0)) * p.H + sq.h) * D);
+          reinterpret_cast<const uint4*>(p.q + (((size_t)sq.b * n + node) * p.H + sq.h * p.group + gi) * D);
 #pragma unroll
       for (int hd = 0; hd < C::kHalves; ++hd)
 #pragma unroll
@@ -367,8 +379,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       if (half == 0 && seg == 0) write_q(s, 0);  // later segments' Q is written ahead (below)
       uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
-      if (valid) {
-        int j = qi;
+      if (valid && p.tree) {  // prefix only: no tree keys, no parent array
+        int j = node;
         for (int step = 0; step < kMaxTree && j >= 0; ++step) {
           anc |= 1ull << j;
           const int pj = p.parent[(size_t)s.b * n + j];
@@ -519,9 +531,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float f1 = other.x == -CUDART_INF_F ? 0.f : fast_exp2(other.x - M);
         const float L = l * f0 + other.y * f1;
         const bool single = s.c_first == s.c_last;
-        const int bh = s.b * p.H + s.h;
-        float* dst = single ? p.out + (((size_t)s.b * n + (valid ? qi : 0)) * p.H + s.h) * D
-                            : partial_slot(p.partials, blockIdx.x + bh, n, D) + (size_t)(valid ? qi : 0) * (D + 2) + 2;
+        const int bh = s.b * p.Hkv + s.h;
+        float* dst = single ? p.out + (((size_t)s.b * n + node) * p.H + s.h * p.group + gi) * D
+                            : partial_slot(p.partials, blockIdx.x + bh, p.rows, D) + (size_t)(valid ? qi : 0) * (D + 2) + 2;
         if (!dead) {
           tc::fence_after_sync();
           const float g0 = single ? f0 / L : f0;
@@ -568,7 +580,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // after this CTA's last tile (see the end of the kernel), so that the
         // merge does not hold up the next segment.  Only the first and the last
         // segment of a CTA's share can be split.
-        if (!single && arrive_split(s, p.H, p.counters, threadIdx.x, 128, last_flag)) {
+        if (!single && arrive_split(s, p.Hkv, p.counters, threadIdx.x, 128, last_flag)) {
           if (sid == 0) pend[npend] = make_int4(s.b, s.h, s.c_first, s.c_last);
           ++npend;
         }
@@ -592,7 +604,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   for (int k = 0; k < np; ++k) {
     Segment s;
     s.b = pend[k].x; s.h = pend[k].y; s.c_first = pend[k].z; s.c_last = pend[k].w;
-    combine_partials(s, p.H, n, D, p.partials, p.counters, p.out, reinterpret_cast<float*>(base + C::off_P),
+    combine_partials(s, p.Hkv, p.rows, D, p.group, p.H, p.partials, p.counters, p.out,
+                     reinterpret_cast<float*>(base + C::off_P),
                      threadIdx.x, kThreads);
   }
 }
@@ -653,10 +666,10 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   int ns = kMaxStages;
   while (ns > 2 && C::smem_bytes(a.B, ns) > (size_t)limit) ns -= 2;
   if (C::smem_bytes(a.B, ns) > (size_t)limit) return cudaErrorNotSupported;
-  const long long rows = (long long)a.B * a.H * a.S_cap;
+  const long long rows = (long long)a.B * a.Hkv * a.S_cap;
   CUtensorMap mk, mv;
   if (!make_kv_map(&mk, a.K, rows, D) || !make_kv_map(&mv, a.V, rows, D)) return cudaErrorNotSupported;
-  const long long tiles_ub = (long long)a.B * a.H * ((a.max_kv_len + a.nq + kTK - 1) / kTK);
+  const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
   long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
@@ -671,6 +684,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
   p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
+  p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.rows = a.nq * p.group; p.tree = a.tree;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
   tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
@@ -681,7 +695,8 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st) {
   if (a.dtype != 0 || (a.D != 128 && a.D != 64)) return cudaErrorNotSupported;
-  if ((long long)a.B * a.H * a.S_cap > 0x7fffffffLL) return cudaErrorNotSupported;  // 32-bit TMA row coordinate
+  if ((long long)a.B * a.Hkv * a.S_cap > 0x7fffffffLL) return cudaErrorNotSupported;  // 32-bit TMA row coordinate
+  if (a.nq * (a.H / a.Hkv) > kM) return cudaErrorNotSupported;  // query rows of a slab beyond one MMA
   if (a.D == 128) return launch_typed<128>(a, st);
   return launch_typed<64>(a, st);
 }

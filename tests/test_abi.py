@@ -36,7 +36,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_abi_version(L):
-    assert gb.glide_abi_version() == 1
+    assert gb.glide_abi_version() == 2
 
 
 def test_status_strings(L):
@@ -156,3 +156,16 @@ def test_spec_sample_rejects(L):
               dict(n=None), dict(t=None), dict(ws=None), dict(wsb=16), dict(lg=FAKE + 4), dict(q=FAKE + 2),
               dict(ws=FAKE + 8)]:
         assert ss(**b) == gb.GLIDE_ERR_INVALID, b
+
+
+def test_grouped_query_descriptors(L):
+    # H_kv must divide H and not exceed it
+    for bad in (dict(H=8, H_kv=3), dict(H=4, H_kv=8), dict(H=4, H_kv=-1)):
+        d = desc(**bad)
+        assert gb.glide_attn_workspace_bytes(d, 1) == 0, bad
+        assert cross(L, d) == gb.GLIDE_ERR_INVALID, bad
+    # 32 query heads over 8 cached heads: 4 rows per node; a 26-node tree needs 104 > 64 rows
+    d = desc(H=32, H_kv=8)
+    assert gb.glide_attn_workspace_bytes(d, 16) > 0 and gb.glide_attn_workspace_bytes(d, 17) == 0
+    assert tree(L, d, n=17) == gb.GLIDE_ERR_UNSUPPORTED
+    assert gb.glide_attn_workspace_bytes(desc(H=128, H_kv=1), 1) == 0      # 128 heads on one cache: > 64 rows
