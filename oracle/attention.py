@@ -160,3 +160,38 @@ def cape_mask(gamma: int, pos: Sequence[int]) -> np.ndarray:
             if (j <= gamma and pos[i] > j) or i == j:
                 keep[i - 1, j - 1] = True
     return keep
+
+
+def block_mask(T: int, L: int) -> np.ndarray:
+    """The training-time block-wise mask of the draft's cross-attention
+    (Section 3.1, "Block-wise Attention Mask"), as printed: entry (j, k) of the
+    T x T attention matrix is kept iff block(j) > block(k), block(x) = the index
+    of x's block of L tokens."""
+    block = np.arange(T) // L
+    return block[:, None] > block[None, :]
+
+
+def block_cross_attn(q: np.ndarray, K: np.ndarray, V: np.ndarray, seq_len: Sequence[int], L: int,
+                     scale: Optional[float] = None, pairs=None) -> np.ndarray:
+    """The draft's cross-attention at training time (Section 3.1): the query of
+    every position j of a training sequence attends to the target's keys and
+    values of the positions k with block(j) > block(k) (the blocks of L tokens
+    before j's own block), so that training sees the delayed cache that
+    speculation sees.  q [B, T, H, D]; K, V [B, H_kv, S_cap, D] hold the
+    target's keys/values of positions 0..T-1; seq_len [B] tokens of each
+    sequence.  A position with nothing to attend to (the first block) and a
+    position at or past seq_len get zeros.  -> out [B, T, H, D]."""
+    B, T, H, D = q.shape
+    sc = 1.0 / np.sqrt(D) if not scale else float(scale)
+    out = np.zeros((B, T, H, D), dtype=np.float64)
+    for b, h in _pairs(B, H, pairs):
+        n = int(seq_len[b])
+        if n == 0:
+            continue
+        hk = kv_head(h, H, K.shape[1])
+        allowed = block_mask(n, L)
+        Kb = widen(K[b, hk, :n])
+        Vb = widen(V[b, hk, :n])
+        Q = widen(q[b, :n, h, :])
+        out[b, :n, h, :] = _softmax_rows_attend((Q @ Kb.T) * sc, allowed, Vb)
+    return out

@@ -719,3 +719,42 @@ def check_gqa_is_repeated_kv(cross_attn, tree_verify_attn):
             o1, o2 = cross_attn(qd, K, V, L), cross_attn(qd, K2, V, L)
             grp = H // H_kv
             assert np.allclose(o1[:, :, :grp], o2[:, :, :grp]) and not np.allclose(o1[:, :, grp:], o2[:, :, grp:])
+
+
+# --------------------------------------------- training-time block mask
+def read_block_golden():
+    lines = [ln.strip() for ln in open(os.path.join(GOLDEN, "block_mask_example.txt"))
+             if ln.strip() and not ln.startswith("#")]
+    T = int(lines[0].split()[1])
+    L = int(lines[1].split()[1])
+    keep = np.array([[c == "1" for c in row] for row in lines[2:]])
+    return T, L, keep
+
+
+def check_block_mask_golden(block_mask):
+    T, L, keep = read_block_golden()
+    assert keep.shape == (T, T)
+    assert np.array_equal(block_mask(T, L), keep), "block mask vs hand-worked example"
+
+
+def check_block_attn_is_delayed_cross(block_cross_attn, cross_attn):
+    """Each position j's training-time output is the inference-time
+    cross-attention of its query over the cache of the blocks before j's own
+    block (kv_len = L * block(j)): the delayed cache the block mask simulates.
+    Positions of the first block, and past a sequence's end, get zeros."""
+    g = _rng(41)
+    for H, H_kv, L in ((4, 4, 5), (4, 2, 3), (2, 1, 7)):
+        B, T, D = 2, 23, 16
+        seq_len = [23, 14]
+        K = g.standard_normal((B, H_kv, T, D)).astype(np.float32)
+        V = g.standard_normal((B, H_kv, T, D)).astype(np.float32)
+        q = g.standard_normal((B, T, H, D)).astype(np.float32)
+        out = block_cross_attn(q, K, V, seq_len, L)
+        for b in range(B):
+            for j in range(T):
+                if j >= seq_len[b] or j < L:
+                    assert np.all(out[b, j] == 0.0), (b, j)
+                    continue
+                kv = L * (j // L)
+                want = cross_attn(q[b:b + 1, j:j + 1], K[b:b + 1], V[b:b + 1], [kv])
+                assert np.allclose(out[b, j], want[0, 0], rtol=1e-12, atol=1e-12), (H, L, b, j)

@@ -398,3 +398,27 @@ def test_mutant_gqa_interleaved_heads(monkeypatch):
     # query head h reading cached head h % H_kv (interleaved) instead of its group's
     monkeypatch.setattr(oatt, "kv_head", lambda h, H, H_kv: h % H_kv)
     _expect_some_fail([lambda: pins.check_gqa_is_repeated_kv(oracle.cross_attn, oracle.tree_verify_attn)])
+
+
+# --------------------------------------------- training-time block mask
+def test_block_mask_golden():
+    pins.check_block_mask_golden(oatt.block_mask)
+
+
+def test_block_attn_is_delayed_cross():
+    pins.check_block_attn_is_delayed_cross(oatt.block_cross_attn, oracle.cross_attn)
+
+
+def test_mutant_block_mask_inclusive(monkeypatch):
+    # a position also seeing its own block (block(j) >= block(k))
+    monkeypatch.setattr(oatt, "block_mask",
+                        lambda T, L: (np.arange(T) // L)[:, None] >= (np.arange(T) // L)[None, :])
+    _expect_some_fail([lambda: pins.check_block_mask_golden(oatt.block_mask),
+                       lambda: pins.check_block_attn_is_delayed_cross(oatt.block_cross_attn, oracle.cross_attn)])
+
+
+def test_mutant_block_mask_causal(monkeypatch):
+    # a plain causal mask (k < j) instead of whole earlier blocks
+    monkeypatch.setattr(oatt, "block_mask", lambda T, L: np.tril(np.ones((T, T), dtype=bool), -1))
+    _expect_some_fail([lambda: pins.check_block_mask_golden(oatt.block_mask),
+                       lambda: pins.check_block_attn_is_delayed_cross(oatt.block_cross_attn, oracle.cross_attn)])
