@@ -55,6 +55,17 @@ def algo_bytes(w: synth.Workload):
     return {"glide_cross_attn": cross, "tree_verify_attn": verify, "tree_accept": accept}
 
 
+def measured_tflops():
+    """Measured dense bf16 TFLOP/s (burst), else the fallback."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        if "bf16_tflops" in d:
+            return float(d["bf16_tflops"])
+    return 1900.0
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -344,8 +355,29 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
     gqa_c_bytes = B * Hk * Lk * w.D * 2 * 2 + B * Hq * w.D * (2 + 4)
     gqa_t_bytes = B * Hk * (Lk + n6) * w.D * 2 * 2 + B * n6 * Hq * w.D * (2 + 4) + 4 * B * (n6 + 1)
     del gK, gV
+    # the draft's training-time cross-attention under the block mask (L = 5) on a
+    # Vicuna-7B training shape: B = 4 sequences of T = 2048, 32 heads, D = 128
+    Bt, Tt, Ht, Lb = 4, 2048, 32, 5
+    tK = torch.randn(Bt, Ht, Tt, w.D, device=dev, dtype=torch.bfloat16)
+    tV = torch.randn_like(tK)
+    tq = torch.randn(Bt, Tt, Ht, w.D, device=dev, dtype=torch.bfloat16)
+    t_out = torch.empty(Bt, Tt, Ht, w.D, device=dev)
+    t_len = torch.full((Bt,), Tt, dtype=torch.int32, device=dev)
+    t_ws = torch.zeros(gb.glide_block_attn_workspace_bytes(gb.make_desc(Bt, Ht, w.D, Tt, gb.GLIDE_BF16), Tt),
+                       dtype=torch.uint8, device=dev)
+    blk_ms = timed(lambda: gb.glide_block_cross_attn(tq, tK, tV, t_len, Lb, t_out, t_ws))
+    vis = sum(Lb * (j // Lb) for j in range(Tt))             # visible (query, key) pairs per (b, h)
+    blk_flops = 4.0 * w.D * vis * Bt * Ht                    # two products, 2 flops per multiply-add
+    blk_bytes = 2 * tK.numel() * 2 + tq.numel() * 2 + t_out.numel() * 4
+    tf_peak = measured_tflops()
+    del tK, tV, tq, t_out, t_ws
     del flush
     return {
+        "block_mask_training_shape": {
+            "avg_us": 1e3 * blk_ms, "tflops": blk_flops / (blk_ms * 1e-3) / 1e12,
+            "frac_of_bf16_peak": blk_flops / (blk_ms * 1e-3) / 1e12 / tf_peak,
+            "gbs_of_compulsory_bytes": blk_bytes / (blk_ms * 1e-3) / 1e9,
+            "shape": f"B={Bt} T={Tt} H={Ht} D={w.D} L={Lb} bf16 (Vicuna-7B training shape)"},
         "gqa_mistral7b_shape": {
             "cross_us": 1e3 * gqa_c_ms, "cross_gbs": gqa_c_bytes / (gqa_c_ms * 1e-3) / 1e9,
             "cross_frac_of_peak": gqa_c_bytes / (gqa_c_ms * 1e-3) / 1e9 / peak,

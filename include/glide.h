@@ -268,6 +268,31 @@ glide_status spec_sample_accept(const int32_t* draft_tokens, const float* draft_
                                 int32_t gamma, int32_t V, int32_t* n_accepted, int32_t* next_token,
                                 void* workspace, size_t workspace_bytes, glide_stream_t stream);
 
+/* Bytes of workspace that glide_block_cross_attn needs for sequences of T
+ * positions; 0 if the descriptor or T is out of range. */
+size_t glide_block_attn_workspace_bytes(const glide_attn_desc* desc, int32_t T);
+
+/*
+ * The draft's cross-attention at training time under the block-wise mask
+ * (Section 3.1, "Block-wise Attention Mask"): the query of every position j of
+ * a training sequence attends to the target's cached keys/values of the
+ * positions k with block(j) > block(k), block(x) = x / L -- the blocks before
+ * j's own, i.e. keys 0 .. L*(j/L)-1 -- so that training sees the delayed cache
+ * that speculation sees:
+ *   out[b,j,h,:] = SoftMax over k < L*(j/L) of (q[b,j,h,:] . K[b,hk,k,:] * scale) V[b,hk,k,:]
+ * with hk = h / (H / H_kv).  Positions of the first block (nothing to attend
+ * to) and positions at or past seq_len[b] get zeros.
+ * q [B,T,H,D] bf16; K_cache/V_cache [B,H_kv,S_cap,D] bf16 holding the target's
+ * keys/values of positions 0..T-1; seq_len [B] int32 on the device (clamped to
+ * [0,T]); out [B,T,H,D] fp32.  1 <= T <= S_cap, L >= 1.  fp32 inputs, more than
+ * 64 query heads per cached head, or B * ceil(T / (64 / (H / H_kv))) > 1024:
+ * GLIDE_ERR_UNSUPPORTED.
+ */
+glide_status glide_block_cross_attn(const glide_attn_desc* desc, const void* q, int32_t T, int32_t L,
+                                    const void* K_cache, const void* V_cache, const int32_t* seq_len,
+                                    float* out, void* workspace, size_t workspace_bytes,
+                                    glide_stream_t stream);
+
 /*
  * glide_cross_attn for callers that cannot allocate device memory when they
  * call (the paper has no counterpart; this is a deployment entry point).

@@ -62,6 +62,9 @@ _SIG = {
     "glide_kv_compact": (ctypes.c_int, [ctypes.POINTER(AttnDesc), ctypes.c_int32, ctypes.c_int64, _P, _P, _P,
                                         ctypes.c_int32, _P, _P, _P, _P]),
     "glide_sample_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32]),
+    "glide_block_attn_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(AttnDesc), ctypes.c_int32]),
+    "glide_block_cross_attn": (ctypes.c_int, [ctypes.POINTER(AttnDesc), _P, ctypes.c_int32, ctypes.c_int32, _P, _P,
+                                              _P, _P, _P, ctypes.c_size_t, _P]),
     "spec_sample_accept": (ctypes.c_int, [_P, _P, _P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _P, _P,
                                           _P, ctypes.c_size_t, _P]),
 }
@@ -287,6 +290,28 @@ def spec_sample_accept(draft_tokens: torch.Tensor, draft_probs: torch.Tensor, ta
                                   workspace.data_ptr(), workspace.numel() * workspace.element_size(), _stream(stream))
     _check(st, "spec_sample_accept")
     return n_accepted, next_token
+
+
+def glide_block_attn_workspace_bytes(desc: AttnDesc, T: int) -> int:
+    return int(lib().glide_block_attn_workspace_bytes(ctypes.byref(desc), int(T)))
+
+
+def glide_block_cross_attn(q: torch.Tensor, K_cache: torch.Tensor, V_cache: torch.Tensor, seq_len: torch.Tensor,
+                           L: int, out: torch.Tensor, workspace: torch.Tensor, scale: float = 0.0, max_ctas: int = 0,
+                           stream=None) -> torch.Tensor:
+    """out[B,T,H,D] fp32 <- the draft's training-time cross-attention of q[B,T,H,D] over the
+    target's K/V[B,H_kv,S_cap,D] under the block-wise mask with blocks of L positions."""
+    desc = _cache_desc(q, K_cache, V_cache, scale, 0, max_ctas)
+    T = q.shape[1]
+    if tuple(out.shape) != tuple(q.shape) or out.dtype != torch.float32 or not out.is_contiguous():
+        raise ValueError("out must be contiguous fp32 [B, T, H, D]")
+    if seq_len.dtype != torch.int32 or tuple(seq_len.shape) != (desc.B,):
+        raise TypeError("seq_len must be int32 [B]")
+    st = lib().glide_block_cross_attn(ctypes.byref(desc), q.data_ptr(), T, int(L), K_cache.data_ptr(),
+                                      V_cache.data_ptr(), seq_len.data_ptr(), out.data_ptr(), workspace.data_ptr(),
+                                      workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(st, "glide_block_cross_attn")
+    return out
 
 
 def glide_validate_tree(parent_idx_host, require_root0: bool = True) -> int:

@@ -69,6 +69,8 @@ glide::AttnArgs make_args(const glide_attn_desc* d, const void* q, const void* K
   a.B = d->B; a.H = d->H; a.D = d->D; a.S_cap = d->S_cap; a.nq = nq; a.max_kv_len = max_kv_len;
   a.Hkv = hkv(d);
   a.tree = parent != nullptr ? 1 : 0;
+  a.block_L = 0;
+  a.T = 0;
   a.dtype = d->dtype == GLIDE_BF16 ? 0 : 1;
   a.scale = d->scale > 0.f ? d->scale : 1.0f / sqrtf((float)d->D);
   a.flags = d->flags;
@@ -242,6 +244,45 @@ glide_status spec_sample_accept(const int32_t* draft_tokens, const float* draft_
   a.draft = draft_tokens; a.q = draft_probs; a.logits = target_logits; a.u = uniforms;
   a.B = B; a.gamma = gamma; a.V = V; a.n_acc = n_accepted; a.next_tok = next_token; a.ws = workspace;
   return from_cuda(glide::launch_spec_sample(a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+namespace {
+// Query tiles of the block mask: kMaxTree rows, H / H_kv heads per position.
+int block_tiles(const glide_attn_desc* d, int T) {
+  const int P = glide::kMaxTree / (d->H / hkv(d));
+  return (T + P - 1) / P;
+}
+size_t block_ws_bytes(const glide_attn_desc* d, int T) {
+  const size_t Bp = (size_t)d->B * block_tiles(d, T);
+  const size_t slots = (size_t)glide::kMaxCtas + Bp * hkv(d);
+  return glide::WsLayout::partials_off((int)Bp, d->H) + slots * glide::kMaxTree * (d->D + 2) * sizeof(float);
+}
+}  // namespace
+
+size_t glide_block_attn_workspace_bytes(const glide_attn_desc* desc, int32_t T) {
+  if (!desc_ok(desc) || T < 1 || T > desc->S_cap || desc->H / hkv(desc) > glide::kMaxTree) return 0;
+  if ((long long)desc->B * block_tiles(desc, T) > glide::kMaxBatch) return 0;
+  return block_ws_bytes(desc, T);
+}
+
+glide_status glide_block_cross_attn(const glide_attn_desc* desc, const void* q, int32_t T, int32_t L,
+                                    const void* K_cache, const void* V_cache, const int32_t* seq_len, float* out,
+                                    void* workspace, size_t workspace_bytes, glide_stream_t stream) {
+  if (!desc_ok(desc)) return GLIDE_ERR_INVALID;
+  if (T < 1 || T > desc->S_cap || L < 1) return GLIDE_ERR_INVALID;
+  if (!q || !K_cache || !V_cache || !seq_len || !out || !workspace) return GLIDE_ERR_INVALID;
+  if (!aligned16(q) || !aligned16(K_cache) || !aligned16(V_cache) || !aligned16(out) || !aligned16(workspace) ||
+      (reinterpret_cast<uintptr_t>(seq_len) & 3u))
+    return GLIDE_ERR_INVALID;
+  if (desc->dtype != GLIDE_BF16 || desc->H / hkv(desc) > glide::kMaxTree) return GLIDE_ERR_UNSUPPORTED;
+  if ((long long)desc->B * block_tiles(desc, T) > glide::kMaxBatch) return GLIDE_ERR_UNSUPPORTED;
+  if (workspace_bytes < block_ws_bytes(desc, T)) return GLIDE_ERR_INVALID;
+  glide::AttnArgs a = make_args(desc, q, K_cache, V_cache, seq_len, nullptr, out, workspace, 1, T);
+  a.block_L = L;
+  a.T = T;
+  cudaError_t e = glide::launch_tree_attn_tc(a, reinterpret_cast<cudaStream_t>(stream));
+  if (e == cudaErrorNotSupported) return GLIDE_ERR_UNSUPPORTED;
+  return from_cuda(e);
 }
 
 glide_status glide_validate_tree(const int32_t* parent_idx_host, int32_t B, int32_t n, int32_t require_root0) {

@@ -248,8 +248,28 @@ __device__ inline bool arrive_split(const Segment& s, int H, unsigned* counters,
   return *flag != 0;
 }
 
+// Where query row r of slab (b, h) goes in the output (-1: nowhere).  Tree
+// verification and cross-attention: out_row with n = nq / group nodes.  The
+// training-time block mask: slab b is sequence b / nqt, query tile b % nqt of
+// P positions; position j = tile * P + r / group of a sequence of seq_len
+// positions (at most T) lands at row (sequence * T + j) if j < seq_len.
+struct OutMap {
+  int group, Hq;
+  int nqt, P, T;            // block mode when nqt > 0
+  const int* seq_len;
+  __device__ long long row(int b, int h, int r, int nq) const {
+    if (nqt == 0) return (long long)out_row(b, h, r, nq, group, Hq);
+    const int sb = b / nqt, qt = b - sb * nqt, node = r / group;
+    const int j = qt * P + node;
+    int n = seq_len[sb];
+    n = n < 0 ? 0 : (n > T ? T : n);
+    if (j >= n) return -1;
+    return ((long long)sb * T + j) * Hq + (long long)h * group + (r - node * group);
+  }
+};
+
 // Merges every split partial of slab (b, h) = (s.b, s.h) into `out` (query
-// rows placed by out_row) and re-arms
+// rows placed by the OutMap) and re-arms
 // the counter; all `nthreads` threads of the CTA call it (it uses
 // __syncthreads).  scratch: shared memory for (2 + kCombineW) * nq floats.
 // Pass 1, one thread per query row: M = max_c m_c, the weights
@@ -257,7 +277,7 @@ __device__ inline bool arrive_split(const Segment& s, int H, unsigned* counters,
 // thread taking kCombineU of them with every load issued before any use.
 constexpr int kCombineW = 8;   // slots whose weights are kept in shared memory
 constexpr int kCombineU = 3;   // outputs per thread per round
-__device__ inline void combine_partials(const Segment& s, int H, int nq, int D, int group, int Hq,
+__device__ inline void combine_partials(const Segment& s, int H, int nq, int D, const OutMap& om,
                                         const float* partials, unsigned* counters, float* out, float* scratch,
                                         int tid, int nthreads) {
   const int bh = s.b * H + s.h;
@@ -349,8 +369,10 @@ __device__ inline void combine_partials(const Segment& s, int H, int nq, int D, 
       if (it < items) {
         const int r = it / cpr, d0 = (it - r * cpr) * 4;
         const float li = Linv[r];
-        *reinterpret_cast<float4*>(out + out_row(s.b, s.h, r, nq, group, Hq) * D + d0) =
-            make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
+        const long long orow = om.row(s.b, s.h, r, nq);
+        if (orow >= 0)
+          *reinterpret_cast<float4*>(out + orow * D + d0) =
+              make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
       }
     }
   }

@@ -24,6 +24,8 @@ struct AttnArgs {
   int nq;                 // queries per (b, h): 1 for cross-attention, n for the tree
   int Hkv;                // cached (key/value) heads; H % Hkv == 0, H / Hkv query heads per cached head
   int tree;               // 1: the nq tree keys follow the prefix (verification); 0: prefix only
+  int block_L;            // > 0: the training-time block mask with blocks of block_L positions
+  int T;                  // block mask: positions per sequence (queries [B, T, H, D]); kv_len = lengths
   int max_kv_len;
   int dtype;              // 0 bf16, 1 f32
   float scale;            // already resolved (never 0)

@@ -111,6 +111,10 @@ struct TcParams {
   int group;  // query heads per cached head (H / Hkv)
   int rows;   // query rows per slab: n nodes x group heads, node-major, <= 64
   int tree;   // 1: the n tree keys follow the prefix (verification); 0: prefix only
+  // training-time block mask (nqt > 0): slab b is sequence b / nqt, query tile
+  // b % nqt of P positions; position j sees keys < L * (j / L); Bq sequences of
+  // at most T positions, seq_len in kv_len
+  int Bq, nqt, P, T, L;
   int ns;  // K/V stages
   float scale_log2;
 };
@@ -142,6 +146,38 @@ __device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;"
 // has its arrivals.
 __device__ __forceinline__ void ml_release() { asm volatile("bar.arrive 3, 256;" ::: "memory"); }
 __device__ __forceinline__ void ml_acquire() { asm volatile("bar.sync 3, 256;" ::: "memory"); }
+
+// The slab table of the block mask: pseudo-sequence s = (sequence s / nqt,
+// query tile s % nqt); its keys end at the last block boundary before its last
+// position, and every key below its first position's limit is visible to all
+// of its rows (plen).  All threads call it (ends with __syncthreads).
+__device__ inline void build_block_tiles(BatchTiles bt, const int* seq_len, int Bp, int H, int nqt, int P, int T,
+                                         int L, int TK) {
+  for (int s = threadIdx.x; s < Bp; s += blockDim.x) {
+    int n = seq_len[s / nqt];
+    n = n < 0 ? 0 : (n > T ? T : n);
+    const int j0 = (s % nqt) * P;
+    int klen = 0, mlim = 0;
+    if (j0 < n) {
+      const int jl = (j0 + P < n ? j0 + P : n) - 1;
+      klen = L * (jl / L);
+      mlim = L * (j0 / L);
+    }
+    bt.plen[s] = mlim;
+    bt.len[s] = klen;
+    bt.ntiles[s] = (klen + TK - 1) / TK;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long a = 0;
+    for (int s = 0; s < Bp; ++s) {
+      bt.start[s] = a;
+      a += (long long)H * bt.ntiles[s];
+    }
+    bt.start[Bp] = a;
+  }
+  __syncthreads();
+}
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -183,8 +219,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
-  build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);  // __syncthreads inside
-  if (!p.tree) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
+  if (p.nqt > 0) {
+    build_block_tiles(bt, p.kv_len, p.B, p.Hkv, p.nqt, p.P, p.T, p.L, kTK);
+    // positions that see no key (the first block) or lie past their sequence: zeros
+    for (long long rw = (long long)blockIdx.x * blockDim.x + threadIdx.x; rw < (long long)p.Bq * p.T;
+         rw += (long long)gridDim.x * blockDim.x) {
+      const int sb = (int)(rw / p.T), j = (int)(rw - (long long)sb * p.T);
+      int sn = p.kv_len[sb];
+      sn = sn < 0 ? 0 : (sn > p.T ? p.T : sn);
+      if (j < p.L || j >= sn) {
+        float4* o4 = reinterpret_cast<float4*>(p.out + rw * p.H * D);
+        for (int e = 0; e < p.H * D / 4; ++e) o4[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+  } else {
+    build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);  // __syncthreads inside
+  }
+  if (!p.tree && p.nqt == 0) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
     const long long total = (long long)p.B * n * p.H * D;
     for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
          idx += (long long)gridDim.x * blockDim.x)
@@ -220,7 +271,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue = [&](Cursor& c, const CUtensorMap* map, uint64_t* full, uint32_t dst0) {
         const int st = c.i % ns;
         mbar_arrive_expect_tx(&full[st], C::kKVTile);
-        const int row = (c.s.b * p.Hkv + c.s.h) * p.S_cap + c.t * kTK;
+        const int cb = p.nqt > 0 ? c.s.b / p.nqt : c.s.b;  // the cache of a block-mask slab is its sequence's
+        const int row = (cb * p.Hkv + c.s.h) * p.S_cap + c.t * kTK;
         for (int hd = 0; hd < C::kHalves; ++hd)
           tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, row, &full[st], pol);
         ++c.i;
@@ -345,8 +397,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = quarter * 16 + rr;            // MMA row
     const int qi = rr * 4 + quarter;              // the query row of this MMA row
     const bool valid = qi < p.rows;
-    const int node = valid ? qi / p.group : 0;    // its tree node (the draft query for cross-attention)
-    const int gi = valid ? qi - node * p.group : 0;  // its head within the slab's group
+    const int node = valid ? qi / p.group : 0;    // its tree node (or position in a block-mask tile)
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t o_col = C::kTmemO + half * D;
     const int sid = threadIdx.x;                  // 0..255 among the softmax threads
@@ -356,17 +407,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Segment sg's queries into the swizzled Q tile (padding rows are zero);
     // the two threads of a row write chunks 0-3 and 4-7 of each 128-byte atom.
     // Key-half-0 warps only.
+    const OutMap om{p.group, p.H, p.nqt, p.P, p.T, p.kv_len};
+    // this thread's query row of slab (sb, h): its row in q / out (-1: none),
+    // and, under the block mask, the keys it sees (< lim)
+    auto row_at = [&](const Segment& sq, int& lim) -> long long {
+      lim = bt.plen[sq.b];
+      if (!valid) return -1;
+      if (p.nqt > 0) lim = p.L * (((sq.b % p.nqt) * p.P + node) / p.L);
+      return om.row(sq.b, sq.h, qi, p.rows);
+    };
     auto write_q = [&](const Segment& sq, int sg) {
       unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
-      const uint4* src =
-          reinterpret_cast<const uint4*>(p.q + (((size_t)sq.b * n + node) * p.H + sq.h * p.group + gi) * D);
+      int lim_unused;
+      const long long qr = row_at(sq, lim_unused);
+      const uint4* src = reinterpret_cast<const uint4*>(p.q + (qr >= 0 ? qr : 0) * D);
 #pragma unroll
       for (int hd = 0; hd < C::kHalves; ++hd)
 #pragma unroll
         for (int cc = 0; cc < 4; ++cc) {
           const int c = cpar * 4 + cc;
           uint4 v = make_uint4(0u, 0u, 0u, 0u);
-          if (valid) v = src[hd * 8 + c];
+          if (qr >= 0) v = src[hd * 8 + c];
           *reinterpret_cast<uint4*>(qrow + hd * C::kQHalf + ((c ^ (row & 7)) << 4)) = v;
         }
       tc::fence_async_smem();
@@ -376,6 +437,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (long long g = g_begin; g < g_end; ++seg) {
       const Segment s = locate(bt, P, p.B, g, g_end);
       const int plen = bt.plen[s.b], len = bt.len[s.b];
+      int rowlim;  // keys below it are visible to this row (the prefix, or a block-mask limit)
+      const long long orow = row_at(s, rowlim);
 
       if (half == 0 && seg == 0) write_q(s, 0);  // later segments' Q is written ahead (below)
       uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
@@ -420,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
             const int key = key0 + 2 * k;
-            const bool vis = key < plen || (key < len && ((anc >> ((key - plen) & 63)) & 1ull));
+            const bool vis = key < rowlim || (key < len && ((anc >> ((key - plen) & 63)) & 1ull));
             sc[k] = vis ? __uint_as_float(cur[k]) * sl2 : -CUDART_INF_F;
           }
         }
@@ -532,12 +595,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float L = l * f0 + other.y * f1;
         const bool single = s.c_first == s.c_last;
         const int bh = s.b * p.Hkv + s.h;
-        float* dst = single ? p.out + (((size_t)s.b * n + node) * p.H + s.h * p.group + gi) * D
+        float* dst = single ? p.out + (orow >= 0 ? orow : 0) * D
                             : partial_slot(p.partials, blockIdx.x + bh, p.rows, D) + (size_t)(valid ? qi : 0) * (D + 2) + 2;
+        const bool write = single ? orow >= 0 : valid;
         if (!dead) {
           tc::fence_after_sync();
-          const float g0 = single ? f0 / L : f0;
-          const float g1 = single ? f1 / L : f1;
+          const float invL = L > 0.f ? 1.f / L : 0.f;  // a row that saw no key (block mask): zeros
+          const float g0 = single ? f0 * invL : f0;
+          const float g1 = single ? f1 * invL : f1;
 #pragma unroll 1
           for (int c = 0; c < D / 32; ++c) {
             uint32_t a[16], b[16];
@@ -558,7 +623,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float4 q4 = cpar ? make_float4(r0, v[4 * j + 2], r1, v[4 * j + 3])
                                      : make_float4(v[4 * j], r0, v[4 * j + 1], r1);
               float* d4 = dst + c * 32 + 8 * j + 4 * cpar;
-              if (valid) {
+              if (write) {
                 if (single) {
                   *reinterpret_cast<float4*>(d4) = q4;
                 } else {  // a partial row starts 8 bytes into a 16-byte boundary
@@ -604,8 +669,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   for (int k = 0; k < np; ++k) {
     Segment s;
     s.b = pend[k].x; s.h = pend[k].y; s.c_first = pend[k].z; s.c_last = pend[k].w;
-    combine_partials(s, p.Hkv, p.rows, D, p.group, p.H, p.partials, p.counters, p.out,
-                     reinterpret_cast<float*>(base + C::off_P),
+    const OutMap om{p.group, p.H, p.nqt, p.P, p.T, p.kv_len};
+    combine_partials(s, p.Hkv, p.rows, D, om, p.partials, p.counters, p.out, reinterpret_cast<float*>(base + C::off_P),
                      threadIdx.x, kThreads);
   }
 }
@@ -663,13 +728,21 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   }
   // As many K/V stages as the shared memory holds, and an even number: K slot
   // j % ns then only ever carries tiles of one parity, i.e. of one S issuer.
+  // The block mask works on (sequence, query tile) slabs: P positions per tile.
+  const int group = a.H / a.Hkv;
+  const int P = a.block_L > 0 ? kM / group : 0;
+  const int nqt = a.block_L > 0 ? (a.T + P - 1) / P : 0;
+  const int Bp = a.block_L > 0 ? a.B * nqt : a.B;  // entries of the slab table
+  if (Bp > kMaxBatch) return cudaErrorNotSupported;
   int ns = kMaxStages;
-  while (ns > 2 && C::smem_bytes(a.B, ns) > (size_t)limit) ns -= 2;
-  if (C::smem_bytes(a.B, ns) > (size_t)limit) return cudaErrorNotSupported;
+  while (ns > 2 && C::smem_bytes(Bp, ns) > (size_t)limit) ns -= 2;
+  if (C::smem_bytes(Bp, ns) > (size_t)limit) return cudaErrorNotSupported;
   const long long rows = (long long)a.B * a.Hkv * a.S_cap;
   CUtensorMap mk, mv;
   if (!make_kv_map(&mk, a.K, rows, D) || !make_kv_map(&mv, a.V, rows, D)) return cudaErrorNotSupported;
-  const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
+  const long long tiles_ub =
+      a.block_L > 0 ? (long long)Bp * a.Hkv * ((a.T + kTK - 1) / kTK)
+                    : (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
   long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
@@ -682,12 +755,13 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   unsigned char* ws = static_cast<unsigned char*>(a.ws);
   p.status = reinterpret_cast<unsigned*>(ws);
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
-  p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
-  p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
-  p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.rows = a.nq * p.group; p.tree = a.tree;
+  p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(Bp, a.H));
+  p.B = Bp; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.block_L > 0 ? P : a.nq;
+  p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.tree = a.block_L > 0 ? 0 : a.tree;
+  p.Bq = a.B; p.nqt = nqt; p.P = P; p.T = a.T; p.L = a.block_L;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
+  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(Bp, ns), st>>>(mk, mv, p);
   return cudaGetLastError();
 }
 
@@ -696,7 +770,8 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st) {
   if (a.dtype != 0 || (a.D != 128 && a.D != 64)) return cudaErrorNotSupported;
   if ((long long)a.B * a.Hkv * a.S_cap > 0x7fffffffLL) return cudaErrorNotSupported;  // 32-bit TMA row coordinate
-  if (a.nq * (a.H / a.Hkv) > kM) return cudaErrorNotSupported;  // query rows of a slab beyond one MMA
+  if (a.block_L == 0 && a.nq * (a.H / a.Hkv) > kM) return cudaErrorNotSupported;  // rows beyond one MMA
+  if (a.H / a.Hkv > kM) return cudaErrorNotSupported;
   if (a.D == 128) return launch_typed<128>(a, st);
   return launch_typed<64>(a, st);
 }

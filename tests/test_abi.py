@@ -169,3 +169,16 @@ def test_grouped_query_descriptors(L):
     assert gb.glide_attn_workspace_bytes(d, 16) > 0 and gb.glide_attn_workspace_bytes(d, 17) == 0
     assert tree(L, d, n=17) == gb.GLIDE_ERR_UNSUPPORTED
     assert gb.glide_attn_workspace_bytes(desc(H=128, H_kv=1), 1) == 0      # 128 heads on one cache: > 64 rows
+
+
+def test_block_cross_attn_rejects(L):
+    def blk(d=None, q=FAKE, T=100, Lb=5, K=FAKE, V=FAKE, sl=FAKE, out=FAKE, ws=FAKE, wsb=1 << 40):
+        d = d or desc()
+        return L.glide_block_cross_attn(ctypes.byref(d), q, T, Lb, K, V, sl, out, ws, wsb, None)
+    assert gb.glide_block_attn_workspace_bytes(desc(), 100) > 0
+    assert gb.glide_block_attn_workspace_bytes(desc(), 301) == 0
+    for b in [dict(T=0), dict(T=301), dict(Lb=0), dict(q=None), dict(K=None), dict(sl=None), dict(out=None),
+              dict(ws=None), dict(wsb=64), dict(q=FAKE + 8), dict(sl=FAKE + 2)]:
+        assert blk(**b) == gb.GLIDE_ERR_INVALID, b
+    assert blk(d=desc(dtype=gb.GLIDE_F32)) == gb.GLIDE_ERR_UNSUPPORTED
+    assert blk(d=desc(B=1024, S_cap=4096), T=4096) == gb.GLIDE_ERR_UNSUPPORTED   # 1024 x 64 query tiles
