@@ -521,23 +521,27 @@ def run_glide(args, rank, world, local_rank):
     r_b = torch.empty(B, dtype=torch.int32).pin_memory()
     K16, V16 = K.view(torch.int16), V.view(torch.int16)
 
-    s_comp = torch.cuda.current_stream()
+    s_comp = torch.cuda.Stream(device=dev)   # not the legacy default stream: it can be captured
     s_h2d = torch.cuda.Stream(device=dev)
     s_d2h = torch.cuda.Stream(device=dev)
 
-    def e2e_step():
-        """One round through the public API with host buffers: inputs stream in
-        on a copy stream in the order they are needed, each call waits only for
-        its own inputs, and results stream back on a second copy stream."""
+    def e2e_enqueue():
+        """One round through the public API with host buffers, enqueued on
+        s_comp: inputs stream in on a copy stream in the order they are
+        needed, each call waits only for its own inputs, and results stream
+        back on a second copy stream, which s_comp joins at the end."""
+        fork = s_comp.record_event()
+        s_h2d.wait_event(fork)
+        s_d2h.wait_event(fork)
         ev_in = []
         with torch.cuda.stream(s_h2d):
             kv_len.copy_(h_kv, non_blocking=True)
-            for b in range(B):
-                K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tk[b], non_blocking=True)
-                V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tv[b], non_blocking=True)
             for i in range(w.gamma):
                 q_draft[i].view(torch.int16).copy_(h_qd[i], non_blocking=True)
                 ev_in.append(s_h2d.record_event())
+            for b in range(B):
+                K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tk[b], non_blocking=True)
+                V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tv[b], non_blocking=True)
             q_tree.view(torch.int16).copy_(h_qt, non_blocking=True)
             parent.copy_(h_par, non_blocking=True)
             ev_tree = s_h2d.record_event()
@@ -565,23 +569,49 @@ def run_glide(args, rank, world, local_rank):
             r_p.copy_(path, non_blocking=True)
             r_l.copy_(ln, non_blocking=True)
             r_b.copy_(bonus, non_blocking=True)
-        s_d2h.synchronize()
+        s_comp.wait_event(s_d2h.record_event())
+        s_comp.wait_event(s_h2d.record_event())
+
+    def eager_step():
+        e2e_enqueue()
         s_comp.synchronize()
 
     h2d = (sum(t.numel() * t.element_size() for t in h_qd) + h_qt.numel() * h_qt.element_size() +
            h_par.numel() * 4 + h_kv.numel() * 4 + h_dr.numel() * 4 + h_lg.numel() * 4 +
            sum(t.numel() * 2 for t in tk) + sum(t.numel() * 2 for t in tv))
     d2h = sum(t.numel() * 4 for t in r_c) + r_t.numel() * 4 + r_p.numel() * 4 + 8 * B
-    for _ in range(2):
-        e2e_step()
-    if world > 1:
-        dist.barrier()
-    e0 = time.perf_counter()
-    for _ in range(e2e_steps):
-        e2e_step()
-    e2e_s = time.perf_counter() - e0
-    e2e_s = max_over_ranks(e2e_s, dev)
+
+    def time_steps(step):
+        for _ in range(2):
+            step()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            step()
+        return max_over_ranks(time.perf_counter() - t0, dev)
+
+    e2e_eager_s = time_steps(eager_step)
+    # The same round captured once as a CUDA graph: every step replays it (all
+    # of its copies and launches) and waits for it, so the host enqueues one
+    # graph instead of ~25 copies and launches between dependent rounds.
+    e2e_launch = "cuda_graph"
+    try:
+        graph = torch.cuda.CUDAGraph()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph, stream=s_comp):
+            e2e_enqueue()
+        torch.cuda.synchronize()
+
+        def graph_step():
+            graph.replay()
+            torch.cuda.current_stream().synchronize()
+        e2e_s = time_steps(graph_step)
+    except Exception as exc:  # capture refused on this stack: the eager round is the number
+        e2e_launch = f"eager (graph capture failed: {type(exc).__name__})"
+        e2e_s = e2e_eager_s
     e2e_value = job_throughput(step_kv * e2e_steps, world, e2e_s) / 1e9
+    e2e_eager = job_throughput(step_kv * e2e_steps, world, e2e_eager_s) / 1e9
 
     # ---- the calls around the round: CaPE expansion (before verification) and
     # the cache update (after acceptance), each timed alone with L2 flushed
@@ -624,7 +654,7 @@ def run_glide(args, rank, world, local_rank):
                 "tree_tokens_per_s_per_layer": tree_tok,
                 "roofline": roof, "kernels": kernels, "next_rows": next_rows, "cpu_baseline": cpu_baseline,
                 "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                        "steps": e2e_steps},
+                        "steps": e2e_steps, "launch": e2e_launch, "eager_value": e2e_eager},
                 "gpu_launches": sum(LAUNCHES_PER_CALL[nm] for nm in names) * args.steps, "clocks": clk}
         if args.force_fma:
             line["config"]["tree_kernel"] = "cuda-core (forced)"
