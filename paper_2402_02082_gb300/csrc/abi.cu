@@ -246,23 +246,9 @@ glide_status spec_sample_accept(const int32_t* draft_tokens, const float* draft_
   return from_cuda(glide::launch_spec_sample(a, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-namespace {
-// Query tiles of the block mask: kMaxTree rows, H / H_kv heads per position.
-int block_tiles(const glide_attn_desc* d, int T) {
-  const int P = glide::kMaxTree / (d->H / hkv(d));
-  return (T + P - 1) / P;
-}
-size_t block_ws_bytes(const glide_attn_desc* d, int T) {
-  const size_t Bp = (size_t)d->B * block_tiles(d, T);
-  const size_t slots = (size_t)glide::kMaxCtas + Bp * hkv(d);
-  return glide::WsLayout::partials_off((int)Bp, d->H) + slots * glide::kMaxTree * (d->D + 2) * sizeof(float);
-}
-}  // namespace
-
 size_t glide_block_attn_workspace_bytes(const glide_attn_desc* desc, int32_t T) {
-  if (!desc_ok(desc) || T < 1 || T > desc->S_cap || desc->H / hkv(desc) > glide::kMaxTree) return 0;
-  if ((long long)desc->B * block_tiles(desc, T) > glide::kMaxBatch) return 0;
-  return block_ws_bytes(desc, T);
+  if (!desc_ok(desc) || T < 1 || T > desc->S_cap) return 0;
+  return glide::WsLayout::kHeader;  // the status word
 }
 
 glide_status glide_block_cross_attn(const glide_attn_desc* desc, const void* q, int32_t T, int32_t L,
@@ -274,13 +260,12 @@ glide_status glide_block_cross_attn(const glide_attn_desc* desc, const void* q, 
   if (!aligned16(q) || !aligned16(K_cache) || !aligned16(V_cache) || !aligned16(out) || !aligned16(workspace) ||
       (reinterpret_cast<uintptr_t>(seq_len) & 3u))
     return GLIDE_ERR_INVALID;
-  if (desc->dtype != GLIDE_BF16 || desc->H / hkv(desc) > glide::kMaxTree) return GLIDE_ERR_UNSUPPORTED;
-  if ((long long)desc->B * block_tiles(desc, T) > glide::kMaxBatch) return GLIDE_ERR_UNSUPPORTED;
-  if (workspace_bytes < block_ws_bytes(desc, T)) return GLIDE_ERR_INVALID;
+  if (desc->dtype != GLIDE_BF16) return GLIDE_ERR_UNSUPPORTED;
+  if (workspace_bytes < glide::WsLayout::kHeader) return GLIDE_ERR_INVALID;
   glide::AttnArgs a = make_args(desc, q, K_cache, V_cache, seq_len, nullptr, out, workspace, 1, T);
   a.block_L = L;
   a.T = T;
-  cudaError_t e = glide::launch_tree_attn_tc(a, reinterpret_cast<cudaStream_t>(stream));
+  cudaError_t e = glide::launch_block_attn(a, reinterpret_cast<cudaStream_t>(stream));
   if (e == cudaErrorNotSupported) return GLIDE_ERR_UNSUPPORTED;
   return from_cuda(e);
 }

@@ -1,0 +1,588 @@
+// The draft's cross-attention at training time under the block-wise mask
+// (Section 3.1, "Block-wise Attention Mask") on the tcgen05 tensor cores.
+//
+// Position j of a training sequence attends to the target's keys and values
+// of the positions k < L * (j / L), the blocks before its own.  Over T
+// positions that is a lower-triangular attention of about T^2 / 2 (query,
+// key) pairs at 4 D flops each: a compute-bound product, unlike the
+// memory-bound decoding kernels.  Both products run on the tensor cores:
+//   S = Q K^T   : M = 128 positions, N = 128 keys, K = D
+//   O += P V    : M = 128, N = D, K = 64 keys, once per key half
+// Operands sit in shared memory in the 128-byte-swizzled K-major layout (Q, K,
+// P) or M/N-major layout (V); accumulators live in tensor memory (TMEM): two
+// S buffers of 128 columns and one O accumulator of D columns per key half.
+//
+// Work item: (sequence b, query head h, tile of 128 positions).  Tile x of a
+// (b, h) sees about x + 1 key tiles, so tile x is paired with tile
+// T/128 - 1 - x and every pair carries the same number of key tiles.  CTA c
+// runs pairs c, c + G, c + 2G, ... in (b, h)-major order: the CTAs that run at
+// the same time read the keys and values of a few heads, which stay in L2.
+//
+// Roles (320 threads, one CTA per SM):
+//   warps 0-7  softmax.  Warp w reads TMEM lane quarter w % 4 (positions
+//              32 (w % 4) .. +31 of the tile, one thread per position) and
+//              key half w / 4 (64 of the tile's 128 keys) with the 32x32b
+//              shape.  Each (position, key half) keeps its own running max
+//              and sum and its own O accumulator, so no value crosses warps
+//              inside the key loop; the halves are merged once per item.
+//   warp 8     producer: lane 0 loads the Q tile of each item and feeds the K
+//              and V rings with 2-D TMA, polling the rings' free slots without
+//              blocking on either.
+//   warp 9     MMA issue (lane 0) and the TMEM allocation.
+//
+// Online softmax in the log2 domain with a lazy reference max: O is rescaled
+// in TMEM only when a tile's max exceeds the reference by more than 8 (factor
+// 256); the final division by the sum taken against the same reference makes
+// the result exact up to rounding.  Keys past the item's last visible key are
+// masked, and their V rows are zeroed in shared memory before P.V (the cache
+// beyond a sequence may hold anything, even NaN); positions at or past the
+// sequence's length are written as zeros whatever their queries hold.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <math_constants.h>
+
+#include "attn_common.cuh"
+#include "kernels.h"
+#include "tc_ptx.cuh"
+#include "tensor_map.h"
+
+namespace glide {
+namespace {
+
+constexpr int kBM = 128;         // positions per work item (MMA rows, TMEM lanes)
+constexpr int kBN = 128;         // keys per tile
+constexpr int kMaxStages = 4;    // K/V ring stages (the launch picks as many as fit)
+constexpr int kSoftWarps = 8;
+constexpr int kProdWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kThreads = 320;
+constexpr int kTmemCols = 512;
+constexpr uint32_t kTmemO = 2 * kBN;  // S buffers at columns 0 and 128, O halves from 256
+constexpr uint32_t kAtom = 128 * 128;  // one 128-byte-swizzle atom of 128 rows
+constexpr float kRescaleLog2 = 8.0f;
+
+constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
+              B_SFREE = 20, B_PFULL = 22, B_PFREE = 23, B_ODONE = 24, B_OFREE = 26, B_MDONE = 27, kNumBars = 28;
+
+template <int D>
+struct BlkCfg {
+  static constexpr int kHalves = D / 64;                // swizzle atoms across the head dim
+  static constexpr uint32_t kQBytes = kHalves * kAtom;  // 128 positions x D
+  static constexpr uint32_t kKV = kHalves * kAtom;      // 128 keys x D
+  static constexpr uint32_t kPBytes = 2 * kAtom;        // 128 positions x 128 keys
+  static constexpr uint32_t off_Q = 0;
+  static constexpr uint32_t off_P = off_Q + kQBytes;
+  static constexpr uint32_t off_K = off_P + kPBytes;
+  static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKV; }
+  static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKV; }
+  static __host__ __device__ uint32_t off_ml(int ns) { return off_bar(ns) + 256; }
+  static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + 2 * 2 * kBM * 8; }
+  static size_t smem_bytes(int ns) { return 1024 + off_misc(ns) + 16; }
+  static_assert(kTmemO + 2 * D <= kTmemCols, "TMEM columns");
+  static_assert(kNumBars * 8 <= 256, "barrier area");
+};
+
+struct BlkParams {
+  float* out;
+  const int* seq_len;
+  unsigned* status;
+  int B, H, Hkv, group, T, S_cap, L;
+  int nqt;             // position tiles per sequence
+  int npb;             // tile pairs per (b, h)
+  long long npairs;    // B * H * npb
+  int ns;              // K/V stages
+  float scale_log2;
+};
+
+// One work item and its keys: positions j0 .. j0+127 of sequence b, query head
+// h; keys [0, klen) are visible to some position of the tile, keys [0, mlim)
+// to every position below the sequence's length n; nt key tiles.
+struct Item {
+  int b, h, j0, n, klen, mlim, nt;
+};
+
+// The items of this CTA in order: pairs blockIdx.x, +G, ...; in each pair the
+// later (larger) tile first.  Items with no visible key are included.
+struct Walker {
+  long long pair;
+  int e;
+  __device__ void start() {
+    pair = blockIdx.x;
+    e = 0;
+  }
+  __device__ bool next(const BlkParams& p, Item& it) {
+    while (pair < p.npairs) {
+      const int k = (int)(pair % p.npb);
+      const long long bh = pair / p.npb;
+      const int qa = p.nqt - 1 - k, qb = k;
+      const int e0 = e;
+      if (e == 0) {
+        e = 1;
+      } else {
+        e = 0;
+        pair += gridDim.x;
+      }
+      if (e0 == 1 && qb >= qa) continue;  // a pair of one tile (the middle of an odd count)
+      it.b = (int)(bh / p.H);
+      it.h = (int)(bh - (long long)it.b * p.H);
+      int n = p.seq_len[it.b];
+      n = n < 0 ? 0 : (n > p.T ? p.T : n);
+      it.n = n;
+      it.j0 = (e0 == 0 ? qa : qb) * kBM;
+      if (it.j0 < n) {
+        const int jl = (it.j0 + kBM < n ? it.j0 + kBM : n) - 1;
+        it.klen = p.L * (jl / p.L);
+        it.mlim = p.L * (it.j0 / p.L);
+      } else {
+        it.klen = 0;
+        it.mlim = 0;
+      }
+      it.nt = (it.klen + kBN - 1) / kBN;
+      return true;
+    }
+    return false;
+  }
+};
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// Warp-uniform bounded wait (see the verification kernel): every lane sees the
+// same outcome, so the warp-collective tcgen05 instructions after it stay
+// convergent.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, unsigned* status) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, status) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Named barrier among the 256 softmax threads.
+__device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    block_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                      const __grid_constant__ CUtensorMap tmV, const BlkParams p) {
+  using C = BlkCfg<D>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const int ns = p.ns;
+  const uint32_t off_V = C::off_V(ns);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(ns));
+  float2* ml = reinterpret_cast<float2*>(base + C::off_ml(ns));  // [item parity][key half][position]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int b = 0; b < kNumBars; ++b) {
+      const bool soft = b == B_SFREE || b == B_SFREE + 1 || b == B_PFULL || b == B_OFREE;
+      mbar_init(&bars[b], soft ? kSoftWarps : 1);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kMmaWarp) {
+    tc::tmem_alloc(tmem_slot, kTmemCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == kProdWarp) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::prefetch_tmap(&tmV);
+      const uint64_t pol_q = policy_evict_first(), pol_kv = policy_evict_last();
+      struct Cursor {  // next tile to load: item it, its tile t, CTA-local tile i, item kq
+        Walker w;
+        Item it;
+        int t, i, kq;
+        bool has, qdone;
+      };
+      auto first = [&](Cursor& c) {  // the next item with keys
+        c.has = false;
+        while (c.w.next(p, c.it))
+          if (c.it.nt > 0) {
+            c.has = true;
+            c.t = 0;
+            c.qdone = false;
+            return;
+          }
+      };
+      auto step = [&](Cursor& c) {
+        ++c.i;
+        if (++c.t == c.it.nt) {
+          ++c.kq;
+          first(c);
+        }
+      };
+      auto kv_row = [&](const Cursor& c) { return (c.it.b * p.Hkv + c.it.h / p.group) * p.S_cap + c.t * kBN; };
+      Cursor ck, cv;
+      ck.w.start();
+      cv.w.start();
+      ck.i = cv.i = ck.kq = cv.kq = 0;
+      first(ck);
+      first(cv);
+      int q_issued = 0;
+      uint64_t t_last = global_timer_ns();
+      int spins = 0, seen = 0;
+      while (ck.has || cv.has) {
+        bool progressed = false;
+        if (ck.has) {
+          if (ck.t == 0 && !ck.qdone) {
+            if (mbar_test_wait(&bars[B_QEMPTY], (ck.kq & 1) ^ 1)) {
+              mbar_arrive_expect_tx(&bars[B_QFULL], C::kQBytes);
+              for (int hd = 0; hd < C::kHalves; ++hd)
+                tc::tma_load_2d(base + C::off_Q + hd * kAtom, &tmQ, ck.it.h * D + hd * 64, ck.it.b * p.T + ck.it.j0,
+                                &bars[B_QFULL], pol_q);
+              ck.qdone = true;
+              ++q_issued;
+              progressed = true;
+            }
+          } else if (mbar_test_wait(&bars[B_KEMPTY + ck.i % ns], ((ck.i / ns) & 1) ^ 1)) {
+            const int st = ck.i % ns;
+            mbar_arrive_expect_tx(&bars[B_KFULL + st], C::kKV);
+            for (int hd = 0; hd < C::kHalves; ++hd)
+              tc::tma_load_2d(base + C::off_K + st * C::kKV + hd * kAtom, &tmK, hd * 64, kv_row(ck),
+                              &bars[B_KFULL + st], pol_kv);
+            step(ck);
+            progressed = true;
+          }
+        }
+        if (cv.has && mbar_test_wait(&bars[B_VEMPTY + cv.i % ns], ((cv.i / ns) & 1) ^ 1)) {
+          const int st = cv.i % ns;
+          mbar_arrive_expect_tx(&bars[B_VFULL + st], C::kKV);
+          for (int hd = 0; hd < C::kHalves; ++hd)
+            tc::tma_load_2d(base + off_V + st * C::kKV + hd * kAtom, &tmV, hd * 64, kv_row(cv), &bars[B_VFULL + st],
+                            pol_kv);
+          step(cv);
+          progressed = true;
+        }
+        if (progressed || ++spins < 64) continue;
+        spins = 0;  // every 64 idle polls: check for an abort or a stall of more than kWaitLimitNs
+        const uint64_t now = global_timer_ns();
+        if (ck.i + cv.i + q_issued != seen) {
+          seen = ck.i + cv.i + q_issued;
+          t_last = now;
+        }
+        if (*abort_flag) break;
+        if (now - t_last > kWaitLimitNs) {
+          *abort_flag = 1;
+          record_status(p.status, kStatusTimeout);
+          break;
+        }
+      }
+      if (ck.has || cv.has) {  // aborted: let issued loads land before the CTA exits
+        for (int j = (ck.i > ns ? ck.i - ns : 0); j < ck.i; ++j) mbar_drain(&bars[B_KFULL + j % ns], (j / ns) & 1);
+        for (int j = (cv.i > ns ? cv.i - ns : 0); j < cv.i; ++j) mbar_drain(&bars[B_VFULL + j % ns], (j / ns) & 1);
+        if (q_issued > 0) mbar_drain(&bars[B_QFULL], (q_issued - 1) & 1);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ----------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(kBM, kBN, false, false);
+      constexpr uint32_t idO = tc::idesc_bf16_f32(kBM, D, false, true);
+      const uint32_t sQ = smem_u32(base + C::off_Q), sP = smem_u32(base + C::off_P);
+      const uint32_t sK = smem_u32(base + C::off_K), sV = smem_u32(base + off_V);
+      bool ok = true;
+      // O_h += P[:, 64h .. 64h+63] V[64h .. 64h+63, :] for key halves h = 0, 1
+      auto issue_pv = [&](int j, bool first_in_item, int kq) -> bool {
+        if (!mbar_wait(&bars[B_PFULL], j & 1, abort_flag, p.status)) return false;
+        if (!mbar_wait(&bars[B_VFULL + j % ns], (j / ns) & 1, abort_flag, p.status)) return false;
+        if (first_in_item && kq > 0 && !mbar_wait(&bars[B_OFREE], (kq - 1) & 1, abort_flag, p.status)) return false;
+        tc::fence_after_sync();
+        const uint32_t vb = sV + (j % ns) * C::kKV;
+#pragma unroll
+        for (int ks = 0; ks < kBN / 16; ++ks) {
+          const int h = ks >> 2;
+          const uint64_t a = tc::sw128_desc(sP + h * kAtom + (ks & 3) * 32, 16, 1024);
+          const uint64_t bdesc = tc::sw128_desc(vb + ks * 16 * 128, kAtom, 1024);
+          tc::mma_bf16(tmem + kTmemO + h * D, a, bdesc, idO, (first_in_item && (ks & 3) == 0) ? 0u : 1u);
+        }
+        tc::mma_commit(&bars[B_PFREE]);
+        tc::mma_commit(&bars[B_VEMPTY + j % ns]);
+        tc::mma_commit(&bars[B_ODONE + (j & 1)]);
+        return true;
+      };
+      Walker w;
+      w.start();
+      Item it;
+      int i = 0, kq = 0;
+      int pend = -1, pend_kq = 0;  // the tile whose P.V is issued after the next S
+      bool pend_first = false;
+      while (ok && w.next(p, it)) {
+        if (it.nt == 0) continue;
+        for (int t = 0; t < it.nt && ok; ++t, ++i) {
+          // At an item's first tile the previous item's last P.V goes first:
+          // this item's S needs its Q tile, which loads only after the
+          // previous item's last S.
+          if (t == 0 && pend >= 0) {
+            ok = issue_pv(pend, pend_first, pend_kq);
+            pend = -1;
+            if (!ok) break;
+          }
+          // S(i) = Q K(i)^T into S buffer i % 2
+          if ((t == 0 && !mbar_wait(&bars[B_QFULL], kq & 1, abort_flag, p.status)) ||
+              !mbar_wait(&bars[B_KFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
+              !mbar_wait(&bars[B_SFREE + (i & 1)], ((i >> 1) & 1) ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          const uint32_t kb = sK + (i % ns) * C::kKV;
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const uint64_t a = tc::sw128_desc(sQ + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
+            const uint64_t bdesc = tc::sw128_desc(kb + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
+            tc::mma_bf16(tmem + (i & 1) * kBN, a, bdesc, idS, ks > 0 ? 1u : 0u);
+          }
+          tc::mma_commit(&bars[B_SFULL + (i & 1)]);
+          tc::mma_commit(&bars[B_KEMPTY + i % ns]);
+          if (t == it.nt - 1) tc::mma_commit(&bars[B_QEMPTY]);
+          if (pend >= 0) ok = issue_pv(pend, pend_first, pend_kq);
+          pend = i;
+          pend_first = t == 0;
+          pend_kq = kq;
+        }
+        ++kq;
+      }
+      if (ok && pend >= 0) issue_pv(pend, pend_first, pend_kq);
+      tc::mma_commit(&bars[B_MDONE]);  // every MMA finished before TMEM is released
+      mbar_drain(&bars[B_MDONE], 0);
+    }
+  } else {
+    // ------------------------------------------------------------- softmax
+    const int quarter = warp & 3, kh = warp >> 2;
+    const int r = quarter * 32 + lane;  // this thread's position in the tile (its TMEM lane)
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    const int sid = threadIdx.x;        // 0..255 among the softmax threads
+    const float sl2 = p.scale_log2;
+    bool dead = false;
+    Walker w;
+    w.start();
+    Item it;
+    int i = 0, kq = 0;
+    while (w.next(p, it)) {
+      const int j = it.j0 + r;
+      const bool in_T = j < p.T;
+      float* orow = p.out + (((size_t)it.b * p.T + (in_T ? j : 0)) * p.H + it.h) * D + kh * (D / 2);
+      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros
+        if (in_T)
+#pragma unroll
+          for (int c = 0; c < D / 8; ++c) reinterpret_cast<float4*>(orow)[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        continue;
+      }
+      const bool valid = j < it.n;
+      const int rowlim = valid ? p.L * (j / p.L) : 0;  // keys below it are visible to this position
+      float m_used = -CUDART_INF_F, l = 0.f;
+      for (int t = 0; t < it.nt; ++t, ++i) {
+        const int sb = i & 1;
+        uint32_t s[64];
+        if (!dead) dead = !warp_wait(&bars[B_SFULL + sb], (i >> 1) & 1, abort_flag, p.status);
+        if (!dead) {
+          tc::fence_after_sync();
+          tc::tmem_ld32(lane_base + sb * kBN + kh * 64, *reinterpret_cast<uint32_t(*)[32]>(s));
+          tc::tmem_ld32(lane_base + sb * kBN + kh * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
+          tc::tmem_wait_ld();
+        } else {
+#pragma unroll
+          for (int e = 0; e < 64; ++e) s[e] = 0u;
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_SFREE + sb]);
+
+        // scores of keys key0 + e in the log2 domain, masked
+        const int key0 = t * kBN + kh * 64;
+        float sc[64];
+        if ((t + 1) * kBN <= it.mlim) {
+#pragma unroll
+          for (int e = 0; e < 64; ++e) sc[e] = __uint_as_float(s[e]) * sl2;
+        } else {
+#pragma unroll
+          for (int e = 0; e < 64; ++e) sc[e] = key0 + e < rowlim ? __uint_as_float(s[e]) * sl2 : -CUDART_INF_F;
+        }
+        float mx[4] = {sc[0], sc[1], sc[2], sc[3]};
+#pragma unroll
+        for (int e = 4; e < 64; ++e) mx[e & 3] = fmaxf(mx[e & 3], sc[e]);
+        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+
+        const bool need = tmax > m_used + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float m_new = need ? tmax : m_used;
+          const float f = need ? fast_exp2(m_used - m_new) : 1.f;
+          l *= f;
+          if (t > 0 && !dead) {  // O holds the P.V of this item's earlier tiles
+            dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 1)], ((i - 1) >> 1) & 1, abort_flag, p.status);
+            if (!dead) {
+              tc::fence_after_sync();
+#pragma unroll 1
+              for (int c = 0; c < D / 32; ++c) {
+                uint32_t o[32];
+                tc::tmem_ld32(lane_base + kTmemO + kh * D + c * 32, o);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * f);
+                tc::tmem_st32(lane_base + kTmemO + kh * D + c * 32, o);
+              }
+              tc::tmem_wait_st();
+            }
+          }
+          m_used = m_new;
+        }
+        const float m_eff = m_used == -CUDART_INF_F ? 0.f : m_used;
+        uint32_t pk[32];
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const float a = fast_exp2(sc[2 * e] - m_eff), b = fast_exp2(sc[2 * e + 1] - m_eff);
+          ls[e & 3] += a + b;
+          pk[e] = pack_bf16x2(a, b);
+        }
+        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+
+        // P row r, key half kh: eight 16-byte chunks of 8 keys, swizzled
+        if (!dead) dead = !warp_wait(&bars[B_PFREE], (i & 1) ^ 1, abort_flag, p.status);
+        {
+          unsigned char* prow = base + C::off_P + kh * kAtom + (r >> 3) * 1024 + (r & 7) * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) =
+                make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        }
+        const int vrows = it.klen - t * kBN;
+        if (vrows < kBN) {  // the item's last tile: clear V rows past its last visible key
+          const int st = i % ns;
+          if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (i / ns) & 1, abort_flag, p.status);
+          if (!dead)
+            for (int idx = sid; idx < (kBN - vrows) * C::kHalves * 8; idx += kSoftWarps * 32) {
+              const int row = vrows + idx / (C::kHalves * 8), rem = idx % (C::kHalves * 8);
+              *reinterpret_cast<uint4*>(base + off_V + st * C::kKV + (rem >> 3) * kAtom + row * 128 + (rem & 7) * 16) =
+                  make_uint4(0u, 0u, 0u, 0u);
+            }
+        }
+        tc::fence_async_smem();
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars[B_PFULL]);
+      }
+
+      // ---- item epilogue: merge the two key halves, O / l into this thread's half of the row
+      const int slot = kq & 1;
+      ml[(slot * 2 + kh) * kBM + r] = make_float2(m_used, l);
+      softmax_sync();
+      const float2 oth = ml[(slot * 2 + (kh ^ 1)) * kBM + r];
+      const float m0 = kh == 0 ? m_used : oth.x, l0 = kh == 0 ? l : oth.y;
+      const float m1 = kh == 0 ? oth.x : m_used, l1 = kh == 0 ? oth.y : l;
+      const float M = fmaxf(m0, m1);
+      const float f0 = m0 == -CUDART_INF_F ? 0.f : fast_exp2(m0 - M);
+      const float f1 = m1 == -CUDART_INF_F ? 0.f : fast_exp2(m1 - M);
+      const float Ls = l0 * f0 + l1 * f1;
+      const bool has_value = valid && Ls > 0.f;  // a position that saw no key, or past the sequence: zeros
+      const float inv = has_value ? 1.f / Ls : 0.f;
+      const int jl = i - 1;
+      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+      if (!dead) {
+        tc::fence_after_sync();
+#pragma unroll 1
+        for (int c = 0; c < D / 64; ++c) {
+          uint32_t a[32], b[32];
+          tc::tmem_ld32(lane_base + kTmemO + kh * (D / 2) + c * 32, a);
+          tc::tmem_ld32(lane_base + kTmemO + D + kh * (D / 2) + c * 32, b);
+          tc::tmem_wait_ld();
+          if (in_T) {
+            float4* dst = reinterpret_cast<float4*>(orow + c * 32);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+              if (has_value)
+                v = make_float4((__uint_as_float(a[4 * e]) * f0 + __uint_as_float(b[4 * e]) * f1) * inv,
+                                (__uint_as_float(a[4 * e + 1]) * f0 + __uint_as_float(b[4 * e + 1]) * f1) * inv,
+                                (__uint_as_float(a[4 * e + 2]) * f0 + __uint_as_float(b[4 * e + 2]) * f1) * inv,
+                                (__uint_as_float(a[4 * e + 3]) * f0 + __uint_as_float(b[4 * e + 3]) * f1) * inv);
+              dst[e] = v;
+            }
+          }
+        }
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_OFREE]);
+      ++kq;
+    }
+  }
+
+  __syncwarp();  // the producer and MMA warps reconverge after their single-lane loops
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+template <int D>
+cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
+  using C = BlkCfg<D>;
+  static bool configured = false;
+  const int limit = smem_optin_bytes();
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(block_attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  int ns = kMaxStages;
+  while (ns > 2 && C::smem_bytes(ns) > (size_t)limit) --ns;
+  if (C::smem_bytes(ns) > (size_t)limit) return cudaErrorNotSupported;
+  CUtensorMap mq, mk, mv;
+  const long long kv_rows = (long long)a.B * a.Hkv * a.S_cap;
+  if (!make_bf16_map(&mq, a.q, (long long)a.B * a.T, (long long)a.H * D, (long long)a.H * D, kBM) ||
+      !make_bf16_map(&mk, a.K, kv_rows, D, D, kBN) || !make_bf16_map(&mv, a.V, kv_rows, D, D, kBN))
+    return cudaErrorNotSupported;
+  BlkParams p;
+  p.out = a.out;
+  p.seq_len = a.kv_len;
+  p.status = reinterpret_cast<unsigned*>(a.ws);
+  p.B = a.B; p.H = a.H; p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.T = a.T; p.S_cap = a.S_cap; p.L = a.block_L;
+  p.nqt = (a.T + kBM - 1) / kBM;
+  p.npb = (p.nqt + 1) / 2;
+  p.npairs = (long long)a.B * a.H * p.npb;
+  p.ns = ns;
+  p.scale_log2 = a.scale * kLog2e;
+  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
+  if (G > p.npairs) G = p.npairs;
+  if (G < 1) G = 1;
+  block_attn_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(ns), st>>>(mq, mk, mv, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_block_attn(const AttnArgs& a, cudaStream_t st) {
+  if (a.dtype != 0 || (a.D != 128 && a.D != 64) || a.block_L < 1 || a.T < 1) return cudaErrorNotSupported;
+  // 32-bit TMA row coordinates, including a tile's reach past the last row
+  if ((long long)a.B * a.T + kBM > 0x7fffffffLL || (long long)a.B * a.Hkv * a.S_cap + kBN > 0x7fffffffLL)
+    return cudaErrorNotSupported;
+  if (a.D == 128) return launch_typed<128>(a, st);
+  return launch_typed<64>(a, st);
+}
+
+}  // namespace glide

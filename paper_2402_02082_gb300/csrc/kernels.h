@@ -88,6 +88,8 @@ cudaError_t launch_tree_attn_fma(const AttnArgs& a, cudaStream_t st);
 // Returns cudaErrorNotSupported when the tensor-core kernel does not apply to `a`.
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st);
 cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st);
+// Training-time block-mask cross-attention (block_L > 0, T positions per sequence).
+cudaError_t launch_block_attn(const AttnArgs& a, cudaStream_t st);
 
 cudaError_t launch_cape_expand(const CapeArgs& a, cudaStream_t st);
 cudaError_t launch_kv_compact(const CompactArgs& a, cudaStream_t st);

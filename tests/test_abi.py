@@ -181,4 +181,6 @@ def test_block_cross_attn_rejects(L):
               dict(ws=None), dict(wsb=64), dict(q=FAKE + 8), dict(sl=FAKE + 2)]:
         assert blk(**b) == gb.GLIDE_ERR_INVALID, b
     assert blk(d=desc(dtype=gb.GLIDE_F32)) == gb.GLIDE_ERR_UNSUPPORTED
-    assert blk(d=desc(B=1024, S_cap=4096), T=4096) == gb.GLIDE_ERR_UNSUPPORTED   # 1024 x 64 query tiles
+    # positions beyond 32-bit TMA row coordinates (B * T > 2^31), refused before any GPU call
+    assert blk(d=desc(B=1024, H=1, S_cap=3_000_000), T=3_000_000) == gb.GLIDE_ERR_UNSUPPORTED
+    assert gb.glide_block_attn_workspace_bytes(desc(B=1024, S_cap=4096), 4096) == 256  # the status word only

@@ -28,6 +28,11 @@ def _lib():
     (3, 200, 4, 4, 128, 5, [200, 199, 0], 1000),
     (1, 100, 2, 1, 64, 1, [100], 0),          # L = 1: plain "earlier positions only"
     (1, 50, 2, 2, 128, 64, [50], 0),          # L > T: every position in the first block
+    (2, 1024, 4, 2, 128, 5, [1024, 901], 0),  # eight position tiles: full and masked key tiles
+    (1, 700, 4, 4, 64, 7, [700], 0),          # D = 64 (four K/V stages), an odd number of tiles
+    (1, 130, 128, 1, 64, 5, [130], 0),        # 128 query heads on one cached head
+    (64, 64, 2, 2, 128, 5, [64] * 63 + [17], 0),  # many sequences of one tile each
+    (2, 640, 2, 2, 128, 5, [640, 640], 2),    # two CTAs walk all ten tile pairs
 ])
 def test_block_cross_attn(B, T, H, H_kv, D, L, seq_len, max_ctas):
     S_cap = (T + 15) // 16 * 16
@@ -49,6 +54,25 @@ def test_block_cross_attn(B, T, H, H_kv, D, L, seq_len, max_ctas):
     live = [(b, h) for b in range(B) for h in range(H) if seq_len[b] > L]
     if live:
         assert_attn_close(got, want, live, f"block mask T{T} H{H}/{H_kv} L{L}")
+
+
+def test_block_cross_attn_rising_scores():
+    """Keys whose norm grows along the sequence push each key tile's maximum
+    score far above the previous ones, so the lazy reference max moves and O
+    is rescaled in tensor memory between tiles of a work item."""
+    B, T, H, D, L = 1, 1024, 2, 128, 5
+    S_cap = T
+    ramp = (1.0 + np.arange(S_cap) / 40.0)[None, None, :, None]
+    K = synth.f32_to_bf16_bits((synth.normal_values(91, 1, (B, H, S_cap, D), "f32") * ramp).astype(np.float32))
+    V = synth.normal_values(91, 2, (B, H, S_cap, D), "bf16")
+    q = synth.normal_values(91, 3, (B, T, H, D), "bf16")
+    desc = gb.make_desc(B, H, D, S_cap, gb.GLIDE_BF16)
+    ws = torch.zeros(gb.glide_block_attn_workspace_bytes(desc, T), dtype=torch.uint8, device="cuda")
+    out = torch.full((B, T, H, D), float("nan"), device="cuda")
+    gb.glide_block_cross_attn(dev(q), dev(K), dev(V), dev(np.asarray([T], np.int32)), L, out, ws)
+    torch.cuda.synchronize()
+    want = oracle.block_cross_attn(q, K, V, [T], L)
+    assert_attn_close(out.cpu().numpy(), want, [(0, 0), (0, 1)], "block mask, rising scores")
 
 
 def test_block_cross_attn_matches_inference_cross_attn():
