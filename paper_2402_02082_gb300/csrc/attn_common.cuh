@@ -248,24 +248,11 @@ __device__ inline bool arrive_split(const Segment& s, int H, unsigned* counters,
   return *flag != 0;
 }
 
-// Where query row r of slab (b, h) goes in the output (-1: nowhere).  Tree
-// verification and cross-attention: out_row with n = nq / group nodes.  The
-// training-time block mask: slab b is sequence b / nqt, query tile b % nqt of
-// P positions; position j = tile * P + r / group of a sequence of seq_len
-// positions (at most T) lands at row (sequence * T + j) if j < seq_len.
+// Where query row r of slab (b, h) goes in the output: out_row with nq / group
+// nodes (tree verification and grouped-query cross-attention).
 struct OutMap {
   int group, Hq;
-  int nqt, P, T;            // block mode when nqt > 0
-  const int* seq_len;
-  __device__ long long row(int b, int h, int r, int nq) const {
-    if (nqt == 0) return (long long)out_row(b, h, r, nq, group, Hq);
-    const int sb = b / nqt, qt = b - sb * nqt, node = r / group;
-    const int j = qt * P + node;
-    int n = seq_len[sb];
-    n = n < 0 ? 0 : (n > T ? T : n);
-    if (j >= n) return -1;
-    return ((long long)sb * T + j) * Hq + (long long)h * group + (r - node * group);
-  }
+  __device__ long long row(int b, int h, int r, int nq) const { return (long long)out_row(b, h, r, nq, group, Hq); }
 };
 
 // Merges every split partial of slab (b, h) = (s.b, s.h) into `out` (query
@@ -369,10 +356,8 @@ __device__ inline void combine_partials(const Segment& s, int H, int nq, int D, 
       if (it < items) {
         const int r = it / cpr, d0 = (it - r * cpr) * 4;
         const float li = Linv[r];
-        const long long orow = om.row(s.b, s.h, r, nq);
-        if (orow >= 0)
-          *reinterpret_cast<float4*>(out + orow * D + d0) =
-              make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
+        *reinterpret_cast<float4*>(out + om.row(s.b, s.h, r, nq) * D + d0) =
+            make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
       }
     }
   }

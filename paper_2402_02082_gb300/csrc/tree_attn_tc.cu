@@ -41,15 +41,13 @@
 // V rows past the end of a slab are zeroed in shared memory before P.V (the
 // cache beyond kv_len + n may hold anything, even NaN).
 #include <cuda.h>
-#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <math_constants.h>
-
-#include <mutex>
 
 #include "attn_common.cuh"
 #include "kernels.h"
 #include "tc_ptx.cuh"
+#include "tensor_map.h"
 
 namespace glide {
 namespace {
@@ -111,10 +109,6 @@ struct TcParams {
   int group;  // query heads per cached head (H / Hkv)
   int rows;   // query rows per slab: n nodes x group heads, node-major, <= 64
   int tree;   // 1: the n tree keys follow the prefix (verification); 0: prefix only
-  // training-time block mask (nqt > 0): slab b is sequence b / nqt, query tile
-  // b % nqt of P positions; position j sees keys < L * (j / L); Bq sequences of
-  // at most T positions, seq_len in kv_len
-  int Bq, nqt, P, T, L;
   int ns;  // K/V stages
   float scale_log2;
 };
@@ -146,38 +140,6 @@ __device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;"
 // has its arrivals.
 __device__ __forceinline__ void ml_release() { asm volatile("bar.arrive 3, 256;" ::: "memory"); }
 __device__ __forceinline__ void ml_acquire() { asm volatile("bar.sync 3, 256;" ::: "memory"); }
-
-// The slab table of the block mask: pseudo-sequence s = (sequence s / nqt,
-// query tile s % nqt); its keys end at the last block boundary before its last
-// position, and every key below its first position's limit is visible to all
-// of its rows (plen).  All threads call it (ends with __syncthreads).
-__device__ inline void build_block_tiles(BatchTiles bt, const int* seq_len, int Bp, int H, int nqt, int P, int T,
-                                         int L, int TK) {
-  for (int s = threadIdx.x; s < Bp; s += blockDim.x) {
-    int n = seq_len[s / nqt];
-    n = n < 0 ? 0 : (n > T ? T : n);
-    const int j0 = (s % nqt) * P;
-    int klen = 0, mlim = 0;
-    if (j0 < n) {
-      const int jl = (j0 + P < n ? j0 + P : n) - 1;
-      klen = L * (jl / L);
-      mlim = L * (j0 / L);
-    }
-    bt.plen[s] = mlim;
-    bt.len[s] = klen;
-    bt.ntiles[s] = (klen + TK - 1) / TK;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    long long a = 0;
-    for (int s = 0; s < Bp; ++s) {
-      bt.start[s] = a;
-      a += (long long)H * bt.ntiles[s];
-    }
-    bt.start[Bp] = a;
-  }
-  __syncthreads();
-}
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -219,23 +181,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
-  if (p.nqt > 0) {
-    build_block_tiles(bt, p.kv_len, p.B, p.Hkv, p.nqt, p.P, p.T, p.L, kTK);
-    // positions that see no key (the first block) or lie past their sequence: zeros
-    for (long long rw = (long long)blockIdx.x * blockDim.x + threadIdx.x; rw < (long long)p.Bq * p.T;
-         rw += (long long)gridDim.x * blockDim.x) {
-      const int sb = (int)(rw / p.T), j = (int)(rw - (long long)sb * p.T);
-      int sn = p.kv_len[sb];
-      sn = sn < 0 ? 0 : (sn > p.T ? p.T : sn);
-      if (j < p.L || j >= sn) {
-        float4* o4 = reinterpret_cast<float4*>(p.out + rw * p.H * D);
-        for (int e = 0; e < p.H * D / 4; ++e) o4[e] = make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    }
-  } else {
-    build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);  // __syncthreads inside
-  }
-  if (!p.tree && p.nqt == 0) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
+  build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);  // __syncthreads inside
+  if (!p.tree) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
     const long long total = (long long)p.B * n * p.H * D;
     for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
          idx += (long long)gridDim.x * blockDim.x)
@@ -271,8 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue = [&](Cursor& c, const CUtensorMap* map, uint64_t* full, uint32_t dst0) {
         const int st = c.i % ns;
         mbar_arrive_expect_tx(&full[st], C::kKVTile);
-        const int cb = p.nqt > 0 ? c.s.b / p.nqt : c.s.b;  // the cache of a block-mask slab is its sequence's
-        const int row = (cb * p.Hkv + c.s.h) * p.S_cap + c.t * kTK;
+        const int row = (c.s.b * p.Hkv + c.s.h) * p.S_cap + c.t * kTK;
         for (int hd = 0; hd < C::kHalves; ++hd)
           tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, row, &full[st], pol);
         ++c.i;
@@ -397,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = quarter * 16 + rr;            // MMA row
     const int qi = rr * 4 + quarter;              // the query row of this MMA row
     const bool valid = qi < p.rows;
-    const int node = valid ? qi / p.group : 0;    // its tree node (or position in a block-mask tile)
+    const int node = valid ? qi / p.group : 0;    // its tree node
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t o_col = C::kTmemO + half * D;
     const int sid = threadIdx.x;                  // 0..255 among the softmax threads
@@ -407,13 +353,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Segment sg's queries into the swizzled Q tile (padding rows are zero);
     // the two threads of a row write chunks 0-3 and 4-7 of each 128-byte atom.
     // Key-half-0 warps only.
-    const OutMap om{p.group, p.H, p.nqt, p.P, p.T, p.kv_len};
+    const OutMap om{p.group, p.H};
     // this thread's query row of slab (sb, h): its row in q / out (-1: none),
-    // and, under the block mask, the keys it sees (< lim)
+    // and the prefix keys it sees (< lim)
     auto row_at = [&](const Segment& sq, int& lim) -> long long {
       lim = bt.plen[sq.b];
       if (!valid) return -1;
-      if (p.nqt > 0) lim = p.L * (((sq.b % p.nqt) * p.P + node) / p.L);
       return om.row(sq.b, sq.h, qi, p.rows);
     };
     auto write_q = [&](const Segment& sq, int sg) {
@@ -437,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (long long g = g_begin; g < g_end; ++seg) {
       const Segment s = locate(bt, P, p.B, g, g_end);
       const int plen = bt.plen[s.b], len = bt.len[s.b];
-      int rowlim;  // keys below it are visible to this row (the prefix, or a block-mask limit)
+      int rowlim;  // keys below it are visible to this row (the prefix)
       const long long orow = row_at(s, rowlim);
 
       if (half == 0 && seg == 0) write_q(s, 0);  // later segments' Q is written ahead (below)
@@ -600,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool write = single ? orow >= 0 : valid;
         if (!dead) {
           tc::fence_after_sync();
-          const float invL = L > 0.f ? 1.f / L : 0.f;  // a row that saw no key (block mask): zeros
+          const float invL = L > 0.f ? 1.f / L : 0.f;  // a padding row has no key: zeros
           const float g0 = single ? f0 * invL : f0;
           const float g1 = single ? f1 * invL : f1;
 #pragma unroll 1
@@ -669,57 +614,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   for (int k = 0; k < np; ++k) {
     Segment s;
     s.b = pend[k].x; s.h = pend[k].y; s.c_first = pend[k].z; s.c_last = pend[k].w;
-    const OutMap om{p.group, p.H, p.nqt, p.P, p.T, p.kv_len};
+    const OutMap om{p.group, p.H};
     combine_partials(s, p.Hkv, p.rows, D, om, p.partials, p.counters, p.out, reinterpret_cast<float*>(base + C::off_P),
                      threadIdx.x, kThreads);
   }
 }
 
 // ------------------------------------------------------------------- host
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  });
-  return fn;
-}
-
-// [rows, D] bf16 view of a K or V cache; boxes of 64 head dims x 64 keys, 128-byte swizzle.
-bool make_kv_map(CUtensorMap* m, const void* base, long long rows, int D) {
-  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
-  if (!fn) return false;
-  const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-  const cuuint32_t box[2] = {64, (cuuint32_t)kTK};
-  const cuuint32_t es[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-int smem_optin() {
-  static int cached = -1;
-  if (cached < 0) {
-    int dev = 0, v = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
-      v = 227 * 1024;
-    cached = v;
-  }
-  return cached;
-}
-
 template <int D>
 cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   using C = TcCfg<D>;
   static bool configured = false;
-  const int limit = smem_optin();
+  const int limit = smem_optin_bytes();
   if (!configured) {
     cudaError_t e =
         cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
@@ -728,21 +634,14 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   }
   // As many K/V stages as the shared memory holds, and an even number: K slot
   // j % ns then only ever carries tiles of one parity, i.e. of one S issuer.
-  // The block mask works on (sequence, query tile) slabs: P positions per tile.
   const int group = a.H / a.Hkv;
-  const int P = a.block_L > 0 ? kM / group : 0;
-  const int nqt = a.block_L > 0 ? (a.T + P - 1) / P : 0;
-  const int Bp = a.block_L > 0 ? a.B * nqt : a.B;  // entries of the slab table
-  if (Bp > kMaxBatch) return cudaErrorNotSupported;
   int ns = kMaxStages;
-  while (ns > 2 && C::smem_bytes(Bp, ns) > (size_t)limit) ns -= 2;
-  if (C::smem_bytes(Bp, ns) > (size_t)limit) return cudaErrorNotSupported;
+  while (ns > 2 && C::smem_bytes(a.B, ns) > (size_t)limit) ns -= 2;
+  if (C::smem_bytes(a.B, ns) > (size_t)limit) return cudaErrorNotSupported;
   const long long rows = (long long)a.B * a.Hkv * a.S_cap;
   CUtensorMap mk, mv;
-  if (!make_kv_map(&mk, a.K, rows, D) || !make_kv_map(&mv, a.V, rows, D)) return cudaErrorNotSupported;
-  const long long tiles_ub =
-      a.block_L > 0 ? (long long)Bp * a.Hkv * ((a.T + kTK - 1) / kTK)
-                    : (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
+  if (!make_bf16_map(&mk, a.K, rows, D, D, kTK) || !make_bf16_map(&mv, a.V, rows, D, D, kTK)) return cudaErrorNotSupported;
+  const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
   long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
@@ -755,13 +654,12 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   unsigned char* ws = static_cast<unsigned char*>(a.ws);
   p.status = reinterpret_cast<unsigned*>(ws);
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
-  p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(Bp, a.H));
-  p.B = Bp; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.block_L > 0 ? P : a.nq;
-  p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.tree = a.block_L > 0 ? 0 : a.tree;
-  p.Bq = a.B; p.nqt = nqt; p.P = P; p.T = a.T; p.L = a.block_L;
+  p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
+  p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
+  p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.tree = a.tree;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(Bp, ns), st>>>(mk, mv, p);
+  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
   return cudaGetLastError();
 }
 
@@ -770,8 +668,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st) {
   if (a.dtype != 0 || (a.D != 128 && a.D != 64)) return cudaErrorNotSupported;
   if ((long long)a.B * a.Hkv * a.S_cap > 0x7fffffffLL) return cudaErrorNotSupported;  // 32-bit TMA row coordinate
-  if (a.block_L == 0 && a.nq * (a.H / a.Hkv) > kM) return cudaErrorNotSupported;  // rows beyond one MMA
-  if (a.H / a.Hkv > kM) return cudaErrorNotSupported;
+  if (a.nq * (a.H / a.Hkv) > kM) return cudaErrorNotSupported;  // rows beyond one MMA
   if (a.D == 128) return launch_typed<128>(a, st);
   return launch_typed<64>(a, st);
 }
