@@ -67,7 +67,7 @@ constexpr uint32_t kStage = 4 * 32 * 128;   // epilogue staging: 32 rows x 128 B
 constexpr float kRescaleLog2 = 8.0f;
 // Every kPolyEvery-th pair of exponentials runs on the FMA pipe (exp2_poly2)
 // instead of the MUFU unit, which alone would bound the softmax.
-constexpr int kPolyEvery = 4;
+constexpr int kPolyEvery = 6;
 
 constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 18, B_SFULL = 20,
               B_PFULL = 23, B_BFREE = 26, B_ODONE = 29, B_OFREE = 31, B_MDONE = 32, kNumBars = 34;
