@@ -132,6 +132,47 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+// The ancestor-or-self set (bit j: node j) of `node` in the tree `parent[0..n)`
+// (parent[j] in [0, j) or anything else for a root), for every lane of the
+// warp at once: lane x holds nodes x and x + 32, each with the set A found so
+// far and the next ancestor P not yet in it (A = {x}, P = parent(x) at first);
+// a round of pointer jumping sets A |= A[P] and P = P[P], so six rounds cover
+// the 64 levels a tree of at most 64 nodes can have.  Two coalesced loads and
+// shuffles replace one dependent global load per tree level.  Warp-collective;
+// a lane with want == false gets 0.
+__device__ inline uint64_t ancestors(const int* parent, int n, int node, bool want, int lane) {
+  uint64_t a[2];
+  int q[2];
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int x = lane + 32 * k;
+    const int px = x < n ? parent[x] : -1;
+    a[k] = x < n ? 1ull << x : 0ull;
+    q[k] = (px >= 0 && px < x) ? px : -1;
+  }
+#pragma unroll
+  for (int round = 0; round < 6; ++round) {
+    uint64_t na[2];
+    int nq[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int y = q[k] < 0 ? 0 : q[k];  // every lane shuffles; a root keeps its set
+      const uint64_t ay0 = __shfl_sync(0xffffffffu, a[0], y & 31), ay1 = __shfl_sync(0xffffffffu, a[1], y & 31);
+      const int qy0 = __shfl_sync(0xffffffffu, q[0], y & 31), qy1 = __shfl_sync(0xffffffffu, q[1], y & 31);
+      na[k] = q[k] < 0 ? a[k] : a[k] | (y < 32 ? ay0 : ay1);
+      nq[k] = q[k] < 0 ? -1 : (y < 32 ? qy0 : qy1);
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      a[k] = na[k];
+      q[k] = nq[k];
+    }
+  }
+  const int v = want ? node : 0;
+  const uint64_t r0 = __shfl_sync(0xffffffffu, a[0], v & 31), r1 = __shfl_sync(0xffffffffu, a[1], v & 31);
+  return want ? (v < 32 ? r0 : r1) : 0ull;
+}
+
 // Named barrier among the 256 softmax threads (id 2; id 1 belongs to the split merge).
 __device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
 // Barrier 3 hands the (max, sum) exchange slot back from the key-half-0 warps
@@ -387,14 +428,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       if (half == 0 && seg == 0) write_q(s, 0);  // later segments' Q is written ahead (below)
       uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
-      if (valid && p.tree) {  // prefix only: no tree keys, no parent array
-        int j = node;
-        for (int step = 0; step < kMaxTree && j >= 0; ++step) {
-          anc |= 1ull << j;
-          const int pj = p.parent[(size_t)s.b * n + j];
-          j = (pj >= 0 && pj < j) ? pj : -1;
-        }
-      }
+      if (p.tree) anc = ancestors(p.parent + (size_t)s.b * n, n, node, valid, lane);  // prefix only: no tree keys
 
       float m_used = -CUDART_INF_F, l = 0.f;  // l: this thread's share of the row sum
       // S of the next tile is loaded while this tile's exponentials run (within
