@@ -83,11 +83,11 @@ struct TcCfg {
   static constexpr uint32_t off_Q = 0;
   static constexpr uint32_t off_P = off_Q + kQBytes;
   static constexpr uint32_t off_K = off_P + 2 * kPBytes;
-  // then ns K stages, ns V stages, barriers, (max, sum) of key half 1, misc, batch table
+  // then ns K stages, ns V stages, barriers, (max, sum) of both key halves, misc, batch table
   static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKVTile; }
   static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKVTile; }
   static __host__ __device__ uint32_t off_ml(int ns) { return off_bar(ns) + 512; }
-  static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + kM * 8; }
+  static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + 2 * kM * 8; }
   static __host__ __device__ uint32_t off_tab(int ns) { return off_misc(ns) + 48; }
   static constexpr uint32_t kTmemO = kSBuf * kTK;                  // S buffers at columns 0, 64, 128, 192
   static constexpr uint32_t kTmemCols = kTmemO + 2 * D <= 256 ? 256 : 512;
@@ -175,12 +175,9 @@ __device__ inline uint64_t ancestors(const int* parent, int n, int node, bool wa
 
 // Named barrier among the 256 softmax threads (id 2; id 1 belongs to the split merge).
 __device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
-// Barrier 3 hands the (max, sum) exchange slot back from the key-half-0 warps
-// (arrive, after reading it) to the key-half-1 warps (sync, before writing it
-// for the next segment).  Both sides count the same segments, so every sync
-// has its arrivals.
-__device__ __forceinline__ void ml_release() { asm volatile("bar.arrive 3, 256;" ::: "memory"); }
-__device__ __forceinline__ void ml_acquire() { asm volatile("bar.sync 3, 256;" ::: "memory"); }
+// Barrier 3: every softmax thread has read the other half's (max, sum) of the
+// segment, so both exchange slots may be written again.
+__device__ __forceinline__ void ml_sync() { asm volatile("bar.sync 3, 256;" ::: "memory"); }
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -210,7 +207,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < kNumBars; ++b) {
       uint32_t cnt = 1;
       if ((b >= B_SFREE && b < B_SFREE + kSBuf) || b == B_PFULL || b == B_PFULL + 1) cnt = kSoftWarps;
-      if (b == B_OFREE || b == B_QFULL || b == B_QFULL + 1) cnt = 4;  // the key-half-0 warps
+      if (b == B_OFREE) cnt = kSoftWarps;                  // both halves read O
+      if (b == B_QFULL || b == B_QFULL + 1) cnt = 4;       // the key-half-0 warps write Q
       mbar_init(&bars[b], cnt);
     }
     *abort_flag = 0;
@@ -554,24 +552,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       // epilogue.
       if (half == 0 && s.g_end < g_end) write_q(locate(bt, P, p.B, s.g_end, g_end), seg + 1);
 
-      // ---- segment epilogue: merge the two key halves, then O / l or a split partial
+      // ---- segment epilogue: merge the two key halves, then O / l or a split
+      // partial.  Each half writes half of the head dims, reading both halves'
+      // accumulators there.
       l += __shfl_xor_sync(0xffffffffu, l, 2);  // the row's sum over both threads
-      if (half == 1) {
-        // the next segment's Q is written ahead, so these warps can reach this
-        // point again while the half-0 warps still read the slot
-        if (seg > 0) ml_acquire();
-        if (cpar == 0) ml[row] = make_float2(m_used, l);
-      }
+      if (cpar == 0) ml[half * kM + row] = make_float2(m_used, l);
       softmax_sync();
-      if (half == 0) {
+      const float2 other = ml[(half ^ 1) * kM + row];
+      // every (max, sum) is read before any half can reach the next segment's
+      // epilogue and overwrite its slot (the next segment's Q is written ahead,
+      // so a half can get there early)
+      ml_sync();
+      {
         const int jl = i - 1;
         if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 3)], (jl >> 2) & 1, abort_flag, p.status);
-        const float2 other = ml[row];
-        if (s.g_end < g_end) ml_release();
-        const float M = fmaxf(m_used, other.x);
-        const float f0 = m_used == -CUDART_INF_F ? 0.f : fast_exp2(m_used - M);
-        const float f1 = other.x == -CUDART_INF_F ? 0.f : fast_exp2(other.x - M);
-        const float L = l * f0 + other.y * f1;
+        const float m0 = half == 0 ? m_used : other.x, l0 = half == 0 ? l : other.y;
+        const float m1 = half == 0 ? other.x : m_used, l1 = half == 0 ? other.y : l;
+        const float M = fmaxf(m0, m1);
+        const float f0 = m0 == -CUDART_INF_F ? 0.f : fast_exp2(m0 - M);
+        const float f1 = m1 == -CUDART_INF_F ? 0.f : fast_exp2(m1 - M);
+        const float L = l0 * f0 + l1 * f1;
         const bool single = s.c_first == s.c_last;
         const int bh = s.b * p.Hkv + s.h;
         float* dst = single ? p.out + (orow >= 0 ? orow : 0) * D
@@ -582,15 +582,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float invL = L > 0.f ? 1.f / L : 0.f;  // a padding row has no key: zeros
           const float g0 = single ? f0 * invL : f0;
           const float g1 = single ? f1 * invL : f1;
-#pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t a[16], b[16];
-            tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + c * 32, a);
-            tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + D + c * 32, b);
-            tc::tmem_wait_ld();
+          constexpr int kChunks = D / 64;  // 32-column chunks per half
+          uint32_t a[kChunks][16], b[kChunks][16];
+#pragma unroll
+          for (int cc = 0; cc < kChunks; ++cc) {
+            const int c = half * kChunks + cc;
+            tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + c * 32, a[cc]);
+            tc::tmem_ld16x64b_x16(lane_addr + C::kTmemO + D + c * 32, b[cc]);
+          }
+          tc::tmem_wait_ld();
+#pragma unroll
+          for (int cc = 0; cc < kChunks; ++cc) {
+            const int c = half * kChunks + cc;
             float v[16];
 #pragma unroll
-            for (int k = 0; k < 16; ++k) v[k] = __uint_as_float(a[k]) * g0 + __uint_as_float(b[k]) * g1;
+            for (int k = 0; k < 16; ++k) v[k] = __uint_as_float(a[cc][k]) * g0 + __uint_as_float(b[cc][k]) * g1;
             // The row's two threads hold its even (cpar 0) and odd (cpar 1)
             // columns; one exchange of two values per 8 columns gives each
             // thread 4 consecutive columns: cpar 0 columns 8j..8j+3, cpar 1
@@ -612,7 +618,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
           }
-          if (!single && valid && cpar == 0) {
+          if (!single && valid && cpar == 0 && half == 0) {
             dst[-2] = M;
             dst[-1] = L;
           }
@@ -624,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // after this CTA's last tile (see the end of the kernel), so that the
         // merge does not hold up the next segment.  Only the first and the last
         // segment of a CTA's share can be split.
-        if (!single && arrive_split(s, p.Hkv, p.counters, threadIdx.x, 128, last_flag)) {
+        if (!single && arrive_split(s, p.Hkv, p.counters, sid, kSoftWarps * 32, last_flag)) {
           if (sid == 0) pend[npend] = make_int4(s.b, s.h, s.c_first, s.c_last);
           ++npend;
         }
