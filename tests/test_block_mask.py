@@ -9,7 +9,7 @@ import oracle
 from paper_2402_02082_gb300 import binding as gb
 from paper_2402_02082_gb300 import build, synth
 
-from gpu_util import assert_attn_close, dev
+from gpu_util import assert_attn_close, dev, sample_pairs
 
 pytestmark = pytest.mark.gpu
 
@@ -121,3 +121,24 @@ def test_two_draft_layers():
         torch.cuda.synchronize()
         want = oracle.cross_attn(q, Kall[l - 1], Vall[l - 1], kv)
         assert_attn_close(out.cpu().numpy(), want, None, f"draft layer {m} on target layer {l}")
+
+
+def test_block_cross_attn_bench_shape_sampled():
+    """The bench's training shape at full size (B = 4, T = 2048, 32 heads,
+    D = 128, L = 5: 137 GFLOP), in the launch configuration the bench times,
+    compared with the oracle on sampled (sequence, head) pairs."""
+    B, T, H, D, L = 4, 2048, 32, 128, 5
+    K = synth.normal_values(4242, 1, (B, H, T, D), "bf16")
+    V = synth.normal_values(4242, 2, (B, H, T, D), "bf16")
+    q = synth.normal_values(4242, 3, (B, T, H, D), "bf16")
+    desc = gb.make_desc(B, H, D, T, gb.GLIDE_BF16)
+    ws = torch.zeros(gb.glide_block_attn_workspace_bytes(desc, T), dtype=torch.uint8, device="cuda")
+    out = torch.full((B, T, H, D), float("nan"), device="cuda")
+    gb.glide_block_cross_attn(dev(q), dev(K), dev(V), dev(np.full(B, T, np.int32)), L, out, ws)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy()
+    assert np.isfinite(got).all()
+    pairs = sample_pairs(B, H, 6, seed=7)
+    want = oracle.block_cross_attn(q, K, V, [T] * B, L, pairs=pairs)
+    assert np.all(got[:, :L] == 0.0)
+    assert_attn_close(got, want, pairs, "block mask at the bench shape")

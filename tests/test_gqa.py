@@ -12,7 +12,7 @@ import oracle
 from paper_2402_02082_gb300 import binding as gb
 from paper_2402_02082_gb300 import build, synth
 
-from gpu_util import assert_attn_close, dev
+from gpu_util import assert_attn_close, dev, sample_pairs
 
 pytestmark = pytest.mark.gpu
 
@@ -109,3 +109,25 @@ def test_gqa_equal_heads_is_multi_head():
         torch.cuda.synchronize()
         outs.append(out.cpu().numpy())
     assert np.array_equal(outs[0], outs[1])
+
+
+def test_gqa_bench_shape_sampled():
+    """Grouped-query attention on the bench's Mistral-7B shape at full size
+    (B = 4, 32 query heads over 8 cached heads, D = 128, kv_len 16384, the
+    6-node chain of GliDe with gamma = 5), both calls, compared with the
+    oracle on sampled (sequence, query head) pairs."""
+    B, H, H_kv, D, L, n = 4, 32, 8, 128, 16384, 6
+    K, V, qd, qt, parent = make(B, H, H_kv, D, [L] * B, n, "bf16", seed=4343, tree="chain")
+    S_cap = K.shape[2]
+    ws = ws_for(B, H, H_kv, D, S_cap, n, "bf16")
+    Kd, Vd, kv = dev(K), dev(V), dev(np.full(B, L, np.int32))
+    oc = torch.full((B, 1, H, D), float("nan"), device="cuda")
+    ot = torch.full((B, n, H, D), float("nan"), device="cuda")
+    gb.glide_cross_attn(dev(qd), Kd, Vd, kv, L, oc, ws)
+    gb.tree_verify_attn(dev(qt), dev(parent), Kd, Vd, kv, L, ot, ws)
+    torch.cuda.synchronize()
+    pairs = sample_pairs(B, H, 6, seed=8)
+    assert_attn_close(oc.cpu().numpy(), oracle.cross_attn(qd, K, V, [L] * B, pairs=pairs), pairs,
+                      "GQA cross-attention at the bench shape")
+    assert_attn_close(ot.cpu().numpy(), oracle.tree_verify_attn(qt, parent, K, V, [L] * B, pairs=pairs), pairs,
+                      "GQA verification at the bench shape")
