@@ -7,15 +7,19 @@
 // key) pairs at 4 D flops each: a compute-bound product, unlike the
 // memory-bound decoding kernels.  Both products run on the tensor cores:
 //   S = Q K^T   : M = 128 positions, N = 128 keys, K = D, operands in shared memory
-//   O += P V    : M = 128, N = D, K = 128 keys, P in tensor memory, V in shared memory
+//   O += P V    : M = 128, N = D, K = 64 keys per key half, P in tensor memory, V in shared memory
 // Q and K sit in shared memory in the 128-byte-swizzled K-major layout, V in
-// the M/N-major layout.  Tensor memory (TMEM, 512 columns) holds three S
-// buffers of 128 columns and the O accumulator (D columns).  The softmax
-// overwrites the first 64 columns of its S buffer with P as bf16 pairs, and
-// the P.V product reads P from there: P never passes through shared memory,
-// whose bandwidth the MMA operand reads, the TMA writes and P stores would
-// otherwise share.  S of tile i + 3 reuses the buffer of tile i, so it waits
-// for the completion of P.V of tile i.
+// the M/N-major layout.  Tensor memory (TMEM, 512 columns) holds two S
+// buffers of 128 columns and one O accumulator of D columns per key half.
+// Two softmax groups take the two 64-key halves of every tile, each with its
+// own running max and sum and its own O accumulator, merged once per item:
+// so every SM sub-partition runs two softmax warps, and one warp's loads,
+// maxima and stores overlap the other's exponentials (the MUFU unit is the
+// softmax's bound).  A group overwrites the first 32 columns of its half of
+// the S buffer with P as bf16 pairs and the P.V product reads P from there:
+// P never passes through shared memory, whose bandwidth the MMA operand reads
+// and the TMA writes already share.  S of tile i + 2 reuses the buffer of tile
+// i, so it waits for the completion of P.V of tile i.
 //
 // Work item: (sequence b, query head h, tile of 128 positions).  Tile x of a
 // (b, h) sees about x + 1 key tiles, so tile x is paired with tile
@@ -23,13 +27,15 @@
 // runs pairs c, c + G, c + 2G, ... in (b, h)-major order: the CTAs that run at
 // the same time read the keys and values of a few heads, which stay in L2.
 //
-// Roles (224 threads, one CTA per SM):
-//   warps 0-3  softmax: one thread per position (TMEM lane), 128 keys per
-//              tile, packed f32x2 arithmetic; then the item's epilogue.
-//   warp 4     producer: lane 0 loads the Q tiles (two buffers) and feeds the
-//              K and V rings with 2-D TMA, polling the free slots of both.
-//   warp 5     S issue (lane 0) and the TMEM allocation.
-//   warp 6     P.V issue (lane 0).  Separate issuers keep S of later tiles
+// Roles (352 threads, one CTA per SM):
+//   warps 0-7  softmax, two groups of four: warp w reads TMEM lane quarter
+//              w % 4 (one thread per position) and key half w / 4 of every
+//              tile, with packed f32x2 arithmetic; then the item's epilogue,
+//              each group writing half of the head dims.
+//   warp 8     producer: lane 0 loads the Q tile and feeds the K and V rings
+//              with 2-D TMA, polling the free slots of both.
+//   warp 9     S issue (lane 0) and the TMEM allocation.
+//   warp 10    P.V issue (lane 0).  Separate issuers keep S of later tiles
 //              from queueing behind the wait for this tile's P.
 //
 // Online softmax in the log2 domain with a lazy reference max: O is rescaled
@@ -54,37 +60,35 @@ namespace {
 constexpr int kBM = 128;          // positions per work item (MMA rows, TMEM lanes)
 constexpr int kBN = 128;          // keys per tile
 constexpr int kMaxStages = 4;     // K/V ring stages (the launch picks as many as fit)
-constexpr int kSoftWarps = 4;
-constexpr int kProdWarp = 4;
-constexpr int kSWarp = 5;
-constexpr int kPVWarp = 6;
-constexpr int kThreads = 224;
+constexpr int kSoftWarps = 8;     // two groups of four: the key halves of every tile
+constexpr int kProdWarp = 8;
+constexpr int kSWarp = 9;
+constexpr int kPVWarp = 10;
+constexpr int kThreads = 352;
 constexpr int kTmemCols = 512;
-constexpr int kSBufs = 3;                   // S / P buffers at columns 0, 128, 256
-constexpr uint32_t kTmemO = kSBufs * kBN;   // O accumulator from column 384
+constexpr int kSBufs = 2;                   // S / P buffers at columns 0, 128
+constexpr uint32_t kTmemO = kSBufs * kBN;   // O of key half h from column 256 + h D
 constexpr uint32_t kAtom = 128 * 128;       // one 128-byte-swizzle atom of 128 rows
-constexpr uint32_t kStage = 4 * 32 * 128;   // epilogue staging: 32 rows x 128 B per softmax warp
+constexpr uint32_t kStage = kSoftWarps * 32 * 128;   // epilogue staging: 32 rows x 128 B per softmax warp
 constexpr float kRescaleLog2 = 8.0f;
-// Every kPolyEvery-th pair of exponentials runs on the FMA pipe (exp2_poly2)
-// instead of the MUFU unit, which alone would bound the softmax.
-constexpr int kPolyEvery = 6;
 
-constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 18, B_SFULL = 20,
-              B_PFULL = 23, B_BFREE = 26, B_ODONE = 29, B_OFREE = 31, B_MDONE = 32, kNumBars = 34;
+constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
+              B_PFULL = 20, B_BFREE = 22, B_ODONE = 24, B_OFREE = 26, B_MDONE = 27, kNumBars = 29;
 
 template <int D>
 struct BlkCfg {
   static constexpr int kHalves = D / 64;                // swizzle atoms across the head dim
   static constexpr uint32_t kQBytes = kHalves * kAtom;  // 128 positions x D
   static constexpr uint32_t kKV = kHalves * kAtom;      // 128 keys x D
-  static constexpr uint32_t off_Q = 0;                  // two Q buffers
-  static constexpr uint32_t off_stg = off_Q + 2 * kQBytes;
+  static constexpr uint32_t off_Q = 0;
+  static constexpr uint32_t off_stg = off_Q + kQBytes;
   static constexpr uint32_t off_K = off_stg + kStage;
   static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKV; }
   static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKV; }
-  static __host__ __device__ uint32_t off_misc(int ns) { return off_bar(ns) + 512; }
+  static __host__ __device__ uint32_t off_ml(int ns) { return off_bar(ns) + 512; }
+  static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + 2 * 2 * kBM * 8; }
   static size_t smem_bytes(int ns) { return 1024 + off_misc(ns) + 16; }
-  static_assert(kTmemO + D <= kTmemCols, "TMEM columns");
+  static_assert(kTmemO + 2 * D <= kTmemCols, "TMEM columns");
   static_assert(kNumBars * 8 <= 512, "barrier area");
 };
 
@@ -201,35 +205,11 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return r;
 }
 
-// 2^x for a pair of x <= 8 (the lazy reference max keeps every exponent
-// there) on the FMA pipe: x = n + f with n = round(x), read from the low
-// mantissa bits of x + 1.5 * 2^23, and f in [-1/2, 1/2]; 2^f from a degree-3
-// polynomial (relative-error minimax fit by Remez exchange, written by
-// exp2_poly.py; max relative error 7.5e-5, far below the bf16 rounding of P);
-// n is added to the exponent field.  x is clamped at -126 so the exponent
-// cannot wrap: a masked key (-inf) gets 2^-126 instead of 0, which no sum of
-// a position with a visible key can notice.
-constexpr float kExpC0 = 0.999928074f, kExpC1 = 0.693260985f, kExpC2 = 0.242611122f, kExpC3 = 0.0551716691f;
-constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
-__device__ __forceinline__ uint64_t exp2_poly2(uint64_t x2) {
-  float x0, x1;
-  unf2(x2, x0, x1);
-  const uint64_t xc = f2(fmaxf(x0, -126.f), fmaxf(x1, -126.f));
-  const uint64_t j = fadd2(xc, f2(kRound, kRound));
-  const uint64_t n = fadd2(j, f2(-kRound, -kRound));
-  const uint64_t f = ffma2(n, f2(-1.f, -1.f), xc);
-  uint64_t q = ffma2(f2(kExpC3, kExpC3), f, f2(kExpC2, kExpC2));
-  q = ffma2(q, f, f2(kExpC1, kExpC1));
-  q = ffma2(q, f, f2(kExpC0, kExpC0));
-  float j0, j1, q0, q1;
-  unf2(j, j0, j1);
-  unf2(q, q0, q1);
-  return f2(__uint_as_float(__float_as_uint(q0) + (__float_as_uint(j0) << 23)),
-            __uint_as_float(__float_as_uint(q1) + (__float_as_uint(j1) << 23)));
-}
+// Named barrier among the eight softmax warps (id 0 is __syncthreads).
+__device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 16384 registers
     block_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const BlkParams p) {
   using C = BlkCfg<D>;
@@ -238,6 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ns = p.ns;
   const uint32_t off_V = C::off_V(ns);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(ns));
+  float2* ml = reinterpret_cast<float2*>(base + C::off_ml(ns));  // [item parity][key half][position]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
 
@@ -303,12 +284,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool progressed = false;
         if (ck.has) {
           if (ck.t == 0 && !ck.qdone) {
-            const int qs = ck.kq & 1;
-            if (mbar_test_wait(&bars[B_QEMPTY + qs], ((ck.kq >> 1) & 1) ^ 1)) {
-              mbar_arrive_expect_tx(&bars[B_QFULL + qs], C::kQBytes);
+            if (mbar_test_wait(&bars[B_QEMPTY], (ck.kq & 1) ^ 1)) {
+              mbar_arrive_expect_tx(&bars[B_QFULL], C::kQBytes);
               for (int hd = 0; hd < C::kHalves; ++hd)
-                tc::tma_load_2d(base + C::off_Q + qs * C::kQBytes + hd * kAtom, &tmQ, ck.it.h * D + hd * 64,
-                                ck.it.b * p.T + ck.it.j0, &bars[B_QFULL + qs], pol_q);
+                tc::tma_load_2d(base + C::off_Q + hd * kAtom, &tmQ, ck.it.h * D + hd * 64, ck.it.b * p.T + ck.it.j0,
+                                &bars[B_QFULL], pol_q);
               ck.qdone = true;
               ++q_issued;
               progressed = true;
@@ -353,8 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (ck.has || cv.has) {  // aborted: let issued loads land before the CTA exits
         for (int j = (ck.i > ns ? ck.i - ns : 0); j < ck.i; ++j) mbar_drain(&bars[B_KFULL + j % ns], (j / ns) & 1);
         for (int j = (cv.i > ns ? cv.i - ns : 0); j < cv.i; ++j) mbar_drain(&bars[B_VFULL + j % ns], (j / ns) & 1);
-        for (int q = (q_issued > 2 ? q_issued - 2 : 0); q < q_issued; ++q)
-          mbar_drain(&bars[B_QFULL + (q & 1)], (q >> 1) & 1);
+        if (q_issued > 0) mbar_drain(&bars[B_QFULL], (q_issued - 1) & 1);
       }
     }
   } else if (warp == kSWarp || warp == kPVWarp) {
@@ -375,26 +354,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < it.nt; ++t, ++i) {
           const int bi = i % kSBufs;
           if (s_role) {
-            // S(i) = Q K(i)^T into buffer i % 3, once P.V of tile i - 3 has read that buffer
-            if ((t == 0 && !mbar_wait(&bars[B_QFULL + (kq & 1)], (kq >> 1) & 1, abort_flag, p.status)) ||
+            // S(i) = Q K(i)^T into buffer i % 2, once P.V of tile i - 2 has read that buffer
+            if ((t == 0 && !mbar_wait(&bars[B_QFULL], kq & 1, abort_flag, p.status)) ||
                 !mbar_wait(&bars[B_KFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
                 !mbar_wait(&bars[B_BFREE + bi], ((i / kSBufs) & 1) ^ 1, abort_flag, p.status)) {
               ok = false;
               break;
             }
             tc::fence_after_sync();
-            const uint32_t qb = sQ + (kq & 1) * C::kQBytes, kb = sK + (i % ns) * C::kKV;
+            const uint32_t kb = sK + (i % ns) * C::kKV;
 #pragma unroll
             for (int ks = 0; ks < D / 16; ++ks) {
-              const uint64_t a = tc::sw128_desc(qb + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
+              const uint64_t a = tc::sw128_desc(sQ + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
               const uint64_t bdesc = tc::sw128_desc(kb + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
               tc::mma_bf16(tmem + bi * kBN, a, bdesc, idS, ks > 0 ? 1u : 0u);
             }
             tc::mma_commit(&bars[B_SFULL + bi]);
             tc::mma_commit(&bars[B_KEMPTY + i % ns]);
-            if (t == it.nt - 1) tc::mma_commit(&bars[B_QEMPTY + (kq & 1)]);
+            if (t == it.nt - 1) tc::mma_commit(&bars[B_QEMPTY]);
           } else {
-            // O (+)= P(i) V(i), P from the first 64 columns of buffer i % 3
+            // O_h (+)= P_h(i) V_h(i) for key halves h = 0, 1: P_h in columns 64h .. 64h+31 of buffer i % 2
             const bool first = t == 0;
             if (!mbar_wait(&bars[B_PFULL + bi], (i / kSBufs) & 1, abort_flag, p.status) ||
                 !mbar_wait(&bars[B_VFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
@@ -406,8 +385,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t vb = sV + (i % ns) * C::kKV;
 #pragma unroll
             for (int ks = 0; ks < kBN / 16; ++ks) {
+              const int h = ks >> 2;
               const uint64_t bdesc = tc::sw128_desc(vb + ks * 16 * 128, kAtom, 1024);
-              tc::mma_bf16_ts(tmem + kTmemO, tmem + bi * kBN + ks * 8, bdesc, idO, (first && ks == 0) ? 0u : 1u);
+              tc::mma_bf16_ts(tmem + kTmemO + h * D, tmem + bi * kBN + h * 64 + (ks & 3) * 8, bdesc, idO,
+                              (first && (ks & 3) == 0) ? 0u : 1u);
             }
             tc::mma_commit(&bars[B_VEMPTY + i % ns]);
             tc::mma_commit(&bars[B_ODONE + (i & 1)]);
@@ -422,9 +403,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------- softmax
-    const int r = warp * 32 + lane;  // this thread's position in the tile (its TMEM lane)
-    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-    const int sid = threadIdx.x;     // 0..127 among the softmax threads
+    const int kh = warp >> 2, quarter = warp & 3;
+    const int r = quarter * 32 + lane;  // this thread's position in the tile (its TMEM lane)
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    const uint32_t o_col = kTmemO + kh * D;
+    const int sid = threadIdx.x;        // 0..255 among the softmax threads
+    const int c0 = kh * (D / 2);        // this group's half of the head dims in the output
     const float sl2 = p.scale_log2;
     unsigned char* stg = base + C::off_stg + warp * 4096;  // this warp's 32 rows x 128 B of staging
     bool dead = false;
@@ -435,12 +419,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (w.next(p, it)) {
       if (it.nt == 0) {  // no visible key anywhere in the tile: zeros, four 128-byte rows per store
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c)
+        for (int c = 0; c < D / 64; ++c)
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const int jr = it.j0 + warp * 32 + k * 4 + (lane >> 3);
+            const int jr = it.j0 + quarter * 32 + k * 4 + (lane >> 3);
             if (jr < p.T)
-              *reinterpret_cast<float4*>(p.out + (((size_t)it.b * p.T + jr) * p.H + it.h) * D + c * 32 +
+              *reinterpret_cast<float4*>(p.out + (((size_t)it.b * p.T + jr) * p.H + it.h) * D + c0 + c * 32 +
                                          (lane & 7) * 4) = make_float4(0.f, 0.f, 0.f, 0.f);
           }
         continue;
@@ -451,77 +435,66 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m_used = -CUDART_INF_F, l = 0.f;
       for (int t = 0; t < it.nt; ++t, ++i) {
         const int bi = i % kSBufs;
-        uint32_t s[kBN];
+        uint32_t s[64];
         if (!dead) dead = !warp_wait(&bars[B_SFULL + bi], (i / kSBufs) & 1, abort_flag, p.status);
         if (!dead) {
           tc::fence_after_sync();
-#pragma unroll
-          for (int c = 0; c < kBN / 32; ++c)
-            tc::tmem_ld32(lane_base + bi * kBN + c * 32, *reinterpret_cast<uint32_t(*)[32]>(s + c * 32));
+          tc::tmem_ld32(lane_base + bi * kBN + kh * 64, *reinterpret_cast<uint32_t(*)[32]>(s));
+          tc::tmem_ld32(lane_base + bi * kBN + kh * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(s + 32));
           tc::tmem_wait_ld();
         } else {
 #pragma unroll
-          for (int e = 0; e < kBN; ++e) s[e] = 0u;
+          for (int e = 0; e < 64; ++e) s[e] = 0u;
         }
         // keys at or past this position's limit: -inf (a suffix of the tile)
-        const int nv = rowlim - t * kBN;
-        if ((t + 1) * kBN > it.mlim && __any_sync(0xffffffffu, nv < kBN)) {
+        const int nv = rowlim - t * kBN - kh * 64;
+        if ((t + 1) * kBN > it.mlim && __any_sync(0xffffffffu, nv < 64)) {
 #pragma unroll
-          for (int e = 0; e < kBN; ++e) s[e] = e < nv ? s[e] : 0xff800000u;
+          for (int e = 0; e < 64; ++e) s[e] = e < nv ? s[e] : 0xff800000u;
         }
-        // row max of the raw scores (the scale is positive), then in the log2 domain
         float mx[4] = {__uint_as_float(s[0]), __uint_as_float(s[1]), __uint_as_float(s[2]), __uint_as_float(s[3])};
 #pragma unroll
-        for (int e = 4; e < kBN; e += 8) {
+        for (int e = 4; e < 64; e += 8) {
           mx[0] = fmax3(mx[0], __uint_as_float(s[e]), __uint_as_float(s[e + 1]));
           mx[1] = fmax3(mx[1], __uint_as_float(s[e + 2]), __uint_as_float(s[e + 3]));
-          if (e + 4 < kBN) {
+          if (e + 4 < 64) {
             mx[2] = fmax3(mx[2], __uint_as_float(s[e + 4]), __uint_as_float(s[e + 5]));
             mx[3] = fmax3(mx[3], __uint_as_float(s[e + 6]), __uint_as_float(s[e + 7]));
           }
         }
         const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * sl2;
-
         const bool need = tmax > m_used + kRescaleLog2;
         if (__any_sync(0xffffffffu, need)) {
           const float m_new = need ? tmax : m_used;
           const float f = need ? fast_exp2(m_used - m_new) : 1.f;
           l *= f;
-          if (t > 0 && !dead) {  // O holds the P.V of this item's earlier tiles
+          if (t > 0 && !dead) {  // O_h holds the P.V of this item's earlier tiles
             dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 1)], ((i - 1) >> 1) & 1, abort_flag, p.status);
             if (!dead) {
               tc::fence_after_sync();
 #pragma unroll 1
               for (int c = 0; c < D / 32; ++c) {
                 uint32_t o[32];
-                tc::tmem_ld32(lane_base + kTmemO + c * 32, o);
+                tc::tmem_ld32(lane_base + o_col + c * 32, o);
                 tc::tmem_wait_ld();
 #pragma unroll
                 for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * f);
-                tc::tmem_st32(lane_base + kTmemO + c * 32, o);
+                tc::tmem_st32(lane_base + o_col + c * 32, o);
               }
               tc::tmem_wait_st();
             }
           }
           m_used = m_new;
         }
-        // p = 2^(s * scale * log2(e) - m), summed in fp32 and packed to bf16 pairs
         const float m_eff = m_used == -CUDART_INF_F ? 0.f : m_used;
         const uint64_t sc2 = f2(sl2, sl2), nm2 = f2(-m_eff, -m_eff);
         uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
-        uint32_t pk[kBN / 2];
+        uint32_t pk[32];
 #pragma unroll
-        for (int e = 0; e < kBN / 2; ++e) {
-          const uint64_t x2 = ffma2(f2(__uint_as_float(s[2 * e]), __uint_as_float(s[2 * e + 1])), sc2, nm2);
-          float p0, p1;
-          if (kPolyEvery > 0 && e % kPolyEvery == kPolyEvery - 1) {
-            unf2(exp2_poly2(x2), p0, p1);
-          } else {
-            float x0, x1;
-            unf2(x2, x0, x1);
-            p0 = fast_exp2(x0);
-            p1 = fast_exp2(x1);
-          }
+        for (int e = 0; e < 32; ++e) {
+          float x0, x1;
+          unf2(ffma2(f2(__uint_as_float(s[2 * e]), __uint_as_float(s[2 * e + 1])), sc2, nm2), x0, x1);
+          const float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
           acc[e & 3] = fadd2(acc[e & 3], f2(p0, p1));
           pk[e] = pack_bf16x2(p0, p1);
         }
@@ -531,9 +504,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           unf2(fadd2(acc[2], acc[3]), b0, b1);
           l += (a0 + a1) + (b0 + b1);
         }
-        if (!dead) {  // P over the first 64 columns of this tile's S buffer
-          tc::tmem_st32(lane_base + bi * kBN, *reinterpret_cast<const uint32_t(*)[32]>(pk));
-          tc::tmem_st32(lane_base + bi * kBN + 32, *reinterpret_cast<const uint32_t(*)[32]>(pk + 32));
+        if (!dead) {  // P over the first 32 columns of this half's part of the S buffer
+          tc::tmem_st32(lane_base + bi * kBN + kh * 64, pk);
           tc::tmem_wait_st();
         }
         const int vrows = it.klen - t * kBN;
@@ -553,30 +525,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&bars[B_PFULL + bi]);
       }
 
-      // ---- item epilogue: O / l, 32 columns at a time, staged so that every
-      // store writes four whole 128-byte rows.  O is released at the end: the
-      // next item's first P.V also waits for its P, which these warps write
-      // only after this epilogue.
-      const int jl = i - 1;
+      // ---- item epilogue: merge the key halves; group h writes head dims [h D/2, (h+1) D/2)
+      const int slot = kq & 1;
+      ml[(slot * 2 + kh) * kBM + r] = make_float2(m_used, l);
+      softmax_sync();
+      const float2 oth = ml[(slot * 2 + (kh ^ 1)) * kBM + r];
+      const float m0 = kh == 0 ? m_used : oth.x, l0 = kh == 0 ? l : oth.y;
+      const float m1 = kh == 0 ? oth.x : m_used, l1 = kh == 0 ? oth.y : l;
+      const float M = fmaxf(m0, m1);
+      const float f0 = m0 == -CUDART_INF_F ? 0.f : fast_exp2(m0 - M);
+      const float f1 = m1 == -CUDART_INF_F ? 0.f : fast_exp2(m1 - M);
       const bool has_value = rowlim > 0;  // a position that saw no key, or past the sequence: zeros
-      const float inv = has_value ? 1.f / l : 0.f;
+      const float inv = has_value ? 1.f / (l0 * f0 + l1 * f1) : 0.f;
+      const float g0 = f0 * inv, g1 = f1 * inv;
+      const int jl = i - 1;
       if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
       if (!dead) {
         tc::fence_after_sync();
-        // the load of chunk c + 1 is in flight while chunk c is staged and stored
-        uint32_t o[2][32];
-        tc::tmem_ld32(lane_base + kTmemO, o[0]);
-#pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
+#pragma unroll 1
+        for (int c = 0; c < D / 64; ++c) {
+          uint32_t a[32], b[32];
+          tc::tmem_ld32(lane_base + kTmemO + c0 + c * 32, a);
+          tc::tmem_ld32(lane_base + kTmemO + D + c0 + c * 32, b);
           tc::tmem_wait_ld();
-          if (c + 1 < D / 32) tc::tmem_ld32(lane_base + kTmemO + (c + 1) * 32, o[(c + 1) & 1]);
-          const uint32_t* oc = o[c & 1];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
             if (has_value)
-              v = make_float4(__uint_as_float(oc[4 * e]) * inv, __uint_as_float(oc[4 * e + 1]) * inv,
-                              __uint_as_float(oc[4 * e + 2]) * inv, __uint_as_float(oc[4 * e + 3]) * inv);
+              v = make_float4(__uint_as_float(a[4 * e]) * g0 + __uint_as_float(b[4 * e]) * g1,
+                              __uint_as_float(a[4 * e + 1]) * g0 + __uint_as_float(b[4 * e + 1]) * g1,
+                              __uint_as_float(a[4 * e + 2]) * g0 + __uint_as_float(b[4 * e + 2]) * g1,
+                              __uint_as_float(a[4 * e + 3]) * g0 + __uint_as_float(b[4 * e + 3]) * g1);
             *reinterpret_cast<float4*>(stg + lane * 128 + ((e ^ (lane & 7)) << 4)) = v;
           }
           __syncwarp();
@@ -584,9 +563,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < 8; ++k) {
             const int rr = k * 4 + (lane >> 3), cc = lane & 7;
             const float4 v = *reinterpret_cast<const float4*>(stg + rr * 128 + ((cc ^ (rr & 7)) << 4));
-            const int jr = it.j0 + warp * 32 + rr;
+            const int jr = it.j0 + quarter * 32 + rr;
             if (jr < p.T)
-              *reinterpret_cast<float4*>(p.out + (((size_t)it.b * p.T + jr) * p.H + it.h) * D + c * 32 + cc * 4) = v;
+              *reinterpret_cast<float4*>(p.out + (((size_t)it.b * p.T + jr) * p.H + it.h) * D + c0 + c * 32 + cc * 4) =
+                  v;
           }
           __syncwarp();
         }
