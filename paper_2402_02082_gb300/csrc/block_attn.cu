@@ -69,7 +69,6 @@ constexpr int kTmemCols = 512;
 constexpr int kSBufs = 2;                   // S / P buffers at columns 0, 128
 constexpr uint32_t kTmemO = kSBufs * kBN;   // O of key half h from column 256 + h D
 constexpr uint32_t kAtom = 128 * 128;       // one 128-byte-swizzle atom of 128 rows
-constexpr uint32_t kStage = kSoftWarps * 32 * 128;   // epilogue staging: 32 rows x 128 B per softmax warp
 constexpr float kRescaleLog2 = 8.0f;
 
 constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
@@ -81,25 +80,27 @@ struct BlkCfg {
   static constexpr uint32_t kQBytes = kHalves * kAtom;  // 128 positions x D
   static constexpr uint32_t kKV = kHalves * kAtom;      // 128 keys x D
   static constexpr uint32_t off_Q = 0;
+  // epilogue staging: per softmax warp two boxes of 32 positions x 32 fp32
+  // outputs (4 KB each, 128-byte swizzle); the second also carries the
+  // warp's (max, sum) pairs to its partner of the other key half
+  static constexpr uint32_t kStage = kSoftWarps * 2 * 4096;
   static constexpr uint32_t off_stg = off_Q + kQBytes;
   static constexpr uint32_t off_K = off_stg + kStage;
   static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKV; }
   static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKV; }
-  static __host__ __device__ uint32_t off_ml(int ns) { return off_bar(ns) + 512; }
-  static __host__ __device__ uint32_t off_misc(int ns) { return off_ml(ns) + 2 * 2 * kBM * 8; }
+  static __host__ __device__ uint32_t off_misc(int ns) { return off_bar(ns) + 512; }
   static size_t smem_bytes(int ns) { return 1024 + off_misc(ns) + 16; }
   static_assert(kTmemO + 2 * D <= kTmemCols, "TMEM columns");
   static_assert(kNumBars * 8 <= 512, "barrier area");
 };
 
 struct BlkParams {
-  float* out;
   const int* seq_len;
   unsigned* status;
   int B, H, Hkv, group, T, S_cap, L;
   int nqt;             // position tiles per sequence
   int npb;             // tile pairs per (b, h)
-  long long npairs;    // B * H * npb
+  int npairs;          // B * H * npb (below 2^31)
   int ns;              // K/V stages
   float scale_log2;
 };
@@ -114,16 +115,18 @@ struct Item {
 // The items of this CTA in order: pairs blockIdx.x, +G, ...; in each pair the
 // later (larger) tile first.  Items with no visible key are included.
 struct Walker {
-  long long pair;
-  int e;
+  int pair, e;
+  int cb, cn;  // the last sequence looked up and its clamped length
   __device__ void start() {
     pair = blockIdx.x;
     e = 0;
+    cb = -1;
+    cn = 0;
   }
   __device__ bool next(const BlkParams& p, Item& it) {
     while (pair < p.npairs) {
-      const int k = (int)(pair % p.npb);
-      const long long bh = pair / p.npb;
+      const int k = pair % p.npb;
+      const int bh = pair / p.npb;
       const int qa = p.nqt - 1 - k, qb = k;
       const int e0 = e;
       if (e == 0) {
@@ -133,10 +136,14 @@ struct Walker {
         pair += gridDim.x;
       }
       if (e0 == 1 && qb >= qa) continue;  // a pair of one tile (the middle of an odd count)
-      it.b = (int)(bh / p.H);
-      it.h = (int)(bh - (long long)it.b * p.H);
-      int n = p.seq_len[it.b];
-      n = n < 0 ? 0 : (n > p.T ? p.T : n);
+      it.b = bh / p.H;
+      it.h = bh - it.b * p.H;
+      if (it.b != cb) {  // consecutive pairs mostly share the sequence: one load per change
+        const int n = p.seq_len[it.b];
+        cb = it.b;
+        cn = n < 0 ? 0 : (n > p.T ? p.T : n);
+      }
+      const int n = cn;
       it.n = n;
       it.j0 = (e0 == 0 ? qa : qb) * kBM;
       if (it.j0 < n) {
@@ -205,20 +212,43 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return r;
 }
 
-// Named barrier among the eight softmax warps (id 0 is __syncthreads).
-__device__ __forceinline__ void softmax_sync() { asm volatile("bar.sync 2, 256;" ::: "memory"); }
+// One 32 x 32 fp32 box of this warp's staging (rows of 128 bytes, 16-byte
+// chunk e of row r at chunk e ^ (r & 7): the 128-byte swizzle) to the output
+// at (x, y, z) by a bulk tensor store from lane 0; the staging box stays in
+// use until the store has read it (tc::bulk_wait_read_all).
+__device__ __forceinline__ void store_box(const CUtensorMap* map, const unsigned char* box, int x, int y, int z,
+                                          int lane) {
+  tc::fence_async_smem();  // this lane's shared-memory writes, visible to the bulk copy
+  __syncwarp();
+  if (lane == 0) {
+    tc::tma_store_3d(map, x, y, z, box);
+    tc::bulk_commit();
+  }
+}
+
+// Until the bulk store from this warp's staging box has read it.
+__device__ __forceinline__ void staging_free(int lane) {
+  if (lane == 0) tc::bulk_wait_read_all();
+  __syncwarp();
+}
+
+// Named barrier of the two softmax warps of one TMEM lane quarter (ids 4-7;
+// id 0 is __syncthreads).
+__device__ __forceinline__ void pair_sync(int quarter) {
+  asm volatile("bar.sync %0, 64;" ::"r"(4 + quarter) : "memory");
+}
 
 template <int D>
 __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 16384 registers
     block_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                      const __grid_constant__ CUtensorMap tmV, const BlkParams p) {
+                      const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                      const BlkParams p) {
   using C = BlkCfg<D>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int ns = p.ns;
   const uint32_t off_V = C::off_V(ns);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(ns));
-  float2* ml = reinterpret_cast<float2*>(base + C::off_ml(ns));  // [item parity][key half][position]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
 
@@ -410,23 +440,22 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
     const int sid = threadIdx.x;        // 0..255 among the softmax threads
     const int c0 = kh * (D / 2);        // this group's half of the head dims in the output
     const float sl2 = p.scale_log2;
-    unsigned char* stg = base + C::off_stg + warp * 4096;  // this warp's 32 rows x 128 B of staging
+    unsigned char* stg = base + C::off_stg + warp * 8192;  // this warp's two staging boxes
     bool dead = false;
     Walker w;
     w.start();
     Item it;
     int i = 0, kq = 0;
     while (w.next(p, it)) {
-      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros, four 128-byte rows per store
+      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros
+        staging_free(lane);
 #pragma unroll 1
-        for (int c = 0; c < D / 64; ++c)
+        for (int c = 0; c < D / 64; ++c) {
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const int jr = it.j0 + quarter * 32 + k * 4 + (lane >> 3);
-            if (jr < p.T)
-              *reinterpret_cast<float4*>(p.out + (((size_t)it.b * p.T + jr) * p.H + it.h) * D + c0 + c * 32 +
-                                         (lane & 7) * 4) = make_float4(0.f, 0.f, 0.f, 0.f);
-          }
+          for (int e = 0; e < 8; ++e)
+            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + (e << 4)) = make_float4(0.f, 0.f, 0.f, 0.f);
+          store_box(&tmO, stg + c * 4096, it.h * D + c0 + c * 32, it.j0 + quarter * 32, it.b, lane);
+        }
         continue;
       }
       const int j = it.j0 + r;
@@ -526,10 +555,14 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
       }
 
       // ---- item epilogue: merge the key halves; group h writes head dims [h D/2, (h+1) D/2)
-      const int slot = kq & 1;
-      ml[(slot * 2 + kh) * kBM + r] = make_float2(m_used, l);
-      softmax_sync();
-      const float2 oth = ml[(slot * 2 + (kh ^ 1)) * kBM + r];
+      // (max, sum) of this thread's position through the second staging boxes:
+      // free again once this warp's earlier stores have read them; the second
+      // barrier keeps both boxes unchanged until the partner has read.
+      staging_free(lane);
+      reinterpret_cast<float2*>(stg + 4096)[lane] = make_float2(m_used, l);
+      pair_sync(quarter);
+      const float2 oth = reinterpret_cast<const float2*>(stg + ((warp ^ 4) - warp) * 8192 + 4096)[lane];
+      pair_sync(quarter);
       const float m0 = kh == 0 ? m_used : oth.x, l0 = kh == 0 ? l : oth.y;
       const float m1 = kh == 0 ? oth.x : m_used, l1 = kh == 0 ? oth.y : l;
       const float M = fmaxf(m0, m1);
@@ -556,19 +589,9 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
                               __uint_as_float(a[4 * e + 1]) * g0 + __uint_as_float(b[4 * e + 1]) * g1,
                               __uint_as_float(a[4 * e + 2]) * g0 + __uint_as_float(b[4 * e + 2]) * g1,
                               __uint_as_float(a[4 * e + 3]) * g0 + __uint_as_float(b[4 * e + 3]) * g1);
-            *reinterpret_cast<float4*>(stg + lane * 128 + ((e ^ (lane & 7)) << 4)) = v;
+            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + ((e ^ (lane & 7)) << 4)) = v;
           }
-          __syncwarp();
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const int rr = k * 4 + (lane >> 3), cc = lane & 7;
-            const float4 v = *reinterpret_cast<const float4*>(stg + rr * 128 + ((cc ^ (rr & 7)) << 4));
-            const int jr = it.j0 + quarter * 32 + rr;
-            if (jr < p.T)
-              *reinterpret_cast<float4*>(p.out + (((size_t)it.b * p.T + jr) * p.H + it.h) * D + c0 + c * 32 + cc * 4) =
-                  v;
-          }
-          __syncwarp();
+          store_box(&tmO, stg + c * 4096, it.h * D + c0 + c * 32, it.j0 + quarter * 32, it.b, lane);
         }
       }
       tc::fence_before_sync();
@@ -578,6 +601,7 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
     }
   }
 
+  if (warp < kSoftWarps && lane == 0) tc::bulk_wait_all();  // the output stores have landed
   __syncwarp();  // the producer and MMA warps reconverge after their single-lane loops
   tc::fence_before_sync();
   __syncthreads();
@@ -600,25 +624,26 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   int ns = kMaxStages;
   while (ns > 2 && C::smem_bytes(ns) > (size_t)limit) --ns;
   if (C::smem_bytes(ns) > (size_t)limit) return cudaErrorNotSupported;
-  CUtensorMap mq, mk, mv;
+  CUtensorMap mq, mk, mv, mo;
   const long long kv_rows = (long long)a.B * a.Hkv * a.S_cap;
   if (!make_bf16_map(&mq, a.q, (long long)a.B * a.T, (long long)a.H * D, (long long)a.H * D, kBM) ||
-      !make_bf16_map(&mk, a.K, kv_rows, D, D, kBN) || !make_bf16_map(&mv, a.V, kv_rows, D, D, kBN))
+      !make_bf16_map(&mk, a.K, kv_rows, D, D, kBN) || !make_bf16_map(&mv, a.V, kv_rows, D, D, kBN) ||
+      !make_f32_seq_map(&mo, a.out, a.B, a.T, (long long)a.H * D))
     return cudaErrorNotSupported;
   BlkParams p;
-  p.out = a.out;
   p.seq_len = a.kv_len;
   p.status = reinterpret_cast<unsigned*>(a.ws);
   p.B = a.B; p.H = a.H; p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.T = a.T; p.S_cap = a.S_cap; p.L = a.block_L;
   p.nqt = (a.T + kBM - 1) / kBM;
   p.npb = (p.nqt + 1) / 2;
-  p.npairs = (long long)a.B * a.H * p.npb;
+  if ((long long)a.B * a.H * p.npb > 0x7fffffffLL) return cudaErrorNotSupported;
+  p.npairs = a.B * a.H * p.npb;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
+  int G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > p.npairs) G = p.npairs;
   if (G < 1) G = 1;
-  block_attn_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(ns), st>>>(mq, mk, mv, p);
+  block_attn_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(ns), st>>>(mq, mk, mv, mo, p);
   return cudaGetLastError();
 }
 
@@ -626,6 +651,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 
 cudaError_t launch_block_attn(const AttnArgs& a, cudaStream_t st) {
   if (a.dtype != 0 || (a.D != 128 && a.D != 64) || a.block_L < 1 || a.T < 1) return cudaErrorNotSupported;
+  if (reinterpret_cast<uintptr_t>(a.out) & 15) return cudaErrorNotSupported;  // bulk tensor stores
   // 32-bit TMA row coordinates, including a tile's reach past the last row
   if ((long long)a.B * a.T + kBM > 0x7fffffffLL || (long long)a.B * a.Hkv * a.S_cap + kBN > 0x7fffffffLL)
     return cudaErrorNotSupported;

@@ -42,6 +42,21 @@ inline bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, long
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// A [B, T, row_elems] fp32 tensor (rows of row_elems contiguous elements)
+// written in boxes of 32 elements (128 bytes, one swizzle atom) x 32 rows of
+// one sequence with the 128-byte swizzle; rows at or past T are not written.
+inline bool make_f32_seq_map(CUtensorMap* m, void* base, long long B, long long T, long long row_elems) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)row_elems, (cuuint64_t)T, (cuuint64_t)B};
+  const cuuint64_t strides[2] = {(cuuint64_t)row_elems * 4, (cuuint64_t)(row_elems * T) * 4};
+  const cuuint32_t box[3] = {32, 32, 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
 // Largest dynamic shared memory a block of the current device may opt in to.
 inline int smem_optin_bytes() {
   static int cached = -1;
