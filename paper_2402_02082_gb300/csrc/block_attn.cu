@@ -9,17 +9,24 @@
 //   S = Q K^T   : M = 128 positions, N = 128 keys, K = D, operands in shared memory
 //   O += P V    : M = 128, N = D, K = 64 keys per key half, P in tensor memory, V in shared memory
 // Q and K sit in shared memory in the 128-byte-swizzled K-major layout, V in
-// the M/N-major layout.  Tensor memory (TMEM, 512 columns) holds two S
-// buffers of 128 columns and one O accumulator of D columns per key half.
-// Two softmax groups take the two 64-key halves of every tile, each with its
-// own running max and sum and its own O accumulator, merged once per item:
-// so every SM sub-partition runs two softmax warps, and one warp's loads,
-// maxima and stores overlap the other's exponentials (the MUFU unit is the
-// softmax's bound).  A group overwrites the first 32 columns of its half of
-// the S buffer with P as bf16 pairs and the P.V product reads P from there:
-// P never passes through shared memory, whose bandwidth the MMA operand reads
-// and the TMA writes already share.  S of tile i + 2 reuses the buffer of tile
-// i, so it waits for the completion of P.V of tile i.
+// the M/N-major layout.  Tensor memory (TMEM, 512 columns) holds three S
+// buffers of 128 columns and the O accumulator (D columns).  Two softmax
+// groups take the two 64-key halves of every tile, so every SM sub-partition
+// runs two softmax warps and one warp's loads, maxima and stores overlap the
+// other's exponentials (the MUFU unit is the softmax's bound).  The partners
+// of a lane quarter agree on each tile's row max through one TMEM column of
+// their halves, so both halves share one reference max and accumulate into
+// the one O; each group rescales, and at the end writes, its half of O's
+// columns.  A group overwrites the first 32 columns of its half of the S
+// buffer with P as bf16 pairs and the P.V product reads P from there: P never
+// passes through shared memory, whose bandwidth the MMA operand reads and the
+// TMA writes already share.  S of tile i + 3 reuses the buffer of tile i, so
+// it waits for the completion of P.V of tile i; three buffers keep that wait
+// off the softmax's path.
+//
+// The epilogue stages O / l per warp in two 4 KB boxes of shared memory (the
+// 128-byte swizzle) and writes them with bulk tensor stores, which drain
+// while the warps go on with the next item.
 //
 // Work item: (sequence b, query head h, tile of 128 positions).  Tile x of a
 // (b, h) sees about x + 1 key tiles, so tile x is paired with tile
@@ -66,13 +73,13 @@ constexpr int kSWarp = 9;
 constexpr int kPVWarp = 10;
 constexpr int kThreads = 352;
 constexpr int kTmemCols = 512;
-constexpr int kSBufs = 2;                   // S / P buffers at columns 0, 128
-constexpr uint32_t kTmemO = kSBufs * kBN;   // O of key half h from column 256 + h D
+constexpr int kSBufs = 3;                   // S / P buffers at columns 0, 128, 256
+constexpr uint32_t kTmemO = kSBufs * kBN;   // the O accumulator from column 384
 constexpr uint32_t kAtom = 128 * 128;       // one 128-byte-swizzle atom of 128 rows
 constexpr float kRescaleLog2 = 8.0f;
 
 constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
-              B_PFULL = 20, B_BFREE = 22, B_ODONE = 24, B_OFREE = 26, B_MDONE = 27, kNumBars = 29;
+              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_OFREE = 29, B_MDONE = 30, kNumBars = 32;
 
 template <int D>
 struct BlkCfg {
@@ -90,7 +97,7 @@ struct BlkCfg {
   static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKV; }
   static __host__ __device__ uint32_t off_misc(int ns) { return off_bar(ns) + 512; }
   static size_t smem_bytes(int ns) { return 1024 + off_misc(ns) + 16; }
-  static_assert(kTmemO + 2 * D <= kTmemCols, "TMEM columns");
+  static_assert(kTmemO + D <= kTmemCols, "TMEM columns");
   static_assert(kNumBars * 8 <= 512, "barrier area");
 };
 
@@ -225,6 +232,11 @@ __device__ __forceinline__ void store_box(const CUtensorMap* map, const unsigned
     tc::bulk_commit();
   }
 }
+
+// A shared-memory descriptor advanced by `bytes`: the start address is the
+// descriptor's low field in 16-byte units, and shared addresses stay below
+// 2^18, so the sum never carries out of it.
+__host__ __device__ constexpr uint64_t desc_step(uint32_t bytes) { return bytes >> 4; }
 
 // Until the bulk store from this warp's staging box has read it.
 __device__ __forceinline__ void staging_free(int lane) {
@@ -372,7 +384,7 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
       const bool s_role = warp == kSWarp;
       constexpr uint32_t idS = tc::idesc_bf16_f32(kBM, kBN, false, false);
       constexpr uint32_t idO = tc::idesc_bf16_f32(kBM, D, false, true);
-      const uint32_t sQ = smem_u32(base + C::off_Q);
+      const uint64_t dQ = tc::sw128_desc(smem_u32(base + C::off_Q), 16, 1024);
       const uint32_t sK = smem_u32(base + C::off_K), sV = smem_u32(base + off_V);
       bool ok = true;
       Walker w;
@@ -384,7 +396,7 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
         for (int t = 0; t < it.nt; ++t, ++i) {
           const int bi = i % kSBufs;
           if (s_role) {
-            // S(i) = Q K(i)^T into buffer i % 2, once P.V of tile i - 2 has read that buffer
+            // S(i) = Q K(i)^T into buffer i % 3, once P.V of tile i - 3 has read that buffer
             if ((t == 0 && !mbar_wait(&bars[B_QFULL], kq & 1, abort_flag, p.status)) ||
                 !mbar_wait(&bars[B_KFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
                 !mbar_wait(&bars[B_BFREE + bi], ((i / kSBufs) & 1) ^ 1, abort_flag, p.status)) {
@@ -392,18 +404,18 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
               break;
             }
             tc::fence_after_sync();
-            const uint32_t kb = sK + (i % ns) * C::kKV;
+            const uint64_t dK = tc::sw128_desc(sK + (i % ns) * C::kKV, 16, 1024);
 #pragma unroll
             for (int ks = 0; ks < D / 16; ++ks) {
-              const uint64_t a = tc::sw128_desc(sQ + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
-              const uint64_t bdesc = tc::sw128_desc(kb + (ks >> 2) * kAtom + (ks & 3) * 32, 16, 1024);
-              tc::mma_bf16(tmem + bi * kBN, a, bdesc, idS, ks > 0 ? 1u : 0u);
+              const uint64_t step = desc_step((ks >> 2) * kAtom + (ks & 3) * 32);
+              tc::mma_bf16(tmem + bi * kBN, dQ + step, dK + step, idS, ks > 0 ? 1u : 0u);
             }
             tc::mma_commit(&bars[B_SFULL + bi]);
             tc::mma_commit(&bars[B_KEMPTY + i % ns]);
             if (t == it.nt - 1) tc::mma_commit(&bars[B_QEMPTY]);
           } else {
-            // O_h (+)= P_h(i) V_h(i) for key halves h = 0, 1: P_h in columns 64h .. 64h+31 of buffer i % 2
+            // O (+)= P_0(i) V_0(i) + P_1(i) V_1(i) over the key halves h = 0, 1: P_h in
+            // columns 64h .. 64h+31 of buffer i % 3
             const bool first = t == 0;
             if (!mbar_wait(&bars[B_PFULL + bi], (i / kSBufs) & 1, abort_flag, p.status) ||
                 !mbar_wait(&bars[B_VFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
@@ -412,14 +424,16 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
               break;
             }
             tc::fence_after_sync();
-            const uint32_t vb = sV + (i % ns) * C::kKV;
-#pragma unroll
-            for (int ks = 0; ks < kBN / 16; ++ks) {
-              const int h = ks >> 2;
-              const uint64_t bdesc = tc::sw128_desc(vb + ks * 16 * 128, kAtom, 1024);
-              tc::mma_bf16_ts(tmem + kTmemO + h * D, tmem + bi * kBN + h * 64 + (ks & 3) * 8, bdesc, idO,
-                              (first && (ks & 3) == 0) ? 0u : 1u);
+            const uint64_t dV = tc::sw128_desc(sV + (i % ns) * C::kKV, kAtom, 1024);
+            const uint32_t pcol = tmem + bi * kBN;
+            if (first) {
+              tc::mma_bf16_ts(tmem + kTmemO, pcol, dV, idO, 0u);
+            } else {
+              tc::mma_bf16_ts(tmem + kTmemO, pcol, dV, idO, 1u);
             }
+#pragma unroll
+            for (int ks = 1; ks < kBN / 16; ++ks)
+              tc::mma_bf16_ts(tmem + kTmemO, pcol + (ks >> 2) * 64 + (ks & 3) * 8, dV + desc_step(ks * 16 * 128), idO, 1u);
             tc::mma_commit(&bars[B_VEMPTY + i % ns]);
             tc::mma_commit(&bars[B_ODONE + (i & 1)]);
             tc::mma_commit(&bars[B_BFREE + bi]);
@@ -436,7 +450,7 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
     const int kh = warp >> 2, quarter = warp & 3;
     const int r = quarter * 32 + lane;  // this thread's position in the tile (its TMEM lane)
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
-    const uint32_t o_col = kTmemO + kh * D;
+    const uint32_t o_col = kTmemO + kh * (D / 2);  // this group's half of the O columns
     const int sid = threadIdx.x;        // 0..255 among the softmax threads
     const int c0 = kh * (D / 2);        // this group's half of the head dims in the output
     const float sl2 = p.scale_log2;
@@ -491,18 +505,32 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
             mx[3] = fmax3(mx[3], __uint_as_float(s[e + 6]), __uint_as_float(s[e + 7]));
           }
         }
-        const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * sl2;
+        float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * sl2;
+        // the row max over both key halves: through column 63 of each half,
+        // already read; the pair barrier orders the partner's read after the write
+        if (!dead) {
+          tc::tmem_st1(lane_base + bi * kBN + kh * 64 + 63, __float_as_uint(tmax));
+          tc::tmem_wait_st();
+        }
+        tc::fence_before_sync();
+        pair_sync(quarter);
+        if (!dead) {
+          tc::fence_after_sync();
+          const uint32_t o = tc::tmem_ld1(lane_base + bi * kBN + (kh ^ 1) * 64 + 63);
+          tc::tmem_wait_ld();
+          tmax = fmaxf(tmax, __uint_as_float(o));
+        }
         const bool need = tmax > m_used + kRescaleLog2;
         if (__any_sync(0xffffffffu, need)) {
           const float m_new = need ? tmax : m_used;
           const float f = need ? fast_exp2(m_used - m_new) : 1.f;
           l *= f;
-          if (t > 0 && !dead) {  // O_h holds the P.V of this item's earlier tiles
+          if (t > 0 && !dead) {  // O holds the P.V of this item's earlier tiles: rescale this group's half
             dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 1)], ((i - 1) >> 1) & 1, abort_flag, p.status);
             if (!dead) {
               tc::fence_after_sync();
 #pragma unroll 1
-              for (int c = 0; c < D / 32; ++c) {
+              for (int c = 0; c < D / 64; ++c) {
                 uint32_t o[32];
                 tc::tmem_ld32(lane_base + o_col + c * 32, o);
                 tc::tmem_wait_ld();
@@ -554,41 +582,32 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
         if (lane == 0) mbar_arrive(&bars[B_PFULL + bi]);
       }
 
-      // ---- item epilogue: merge the key halves; group h writes head dims [h D/2, (h+1) D/2)
-      // (max, sum) of this thread's position through the second staging boxes:
-      // free again once this warp's earlier stores have read them; the second
-      // barrier keeps both boxes unchanged until the partner has read.
+      // ---- item epilogue: group h writes head dims [h D/2, (h+1) D/2) of O / l
+      // The partner's sum (taken against the same reference max) through the
+      // second staging boxes: free again once this warp's earlier stores have
+      // read them; the second barrier keeps both unchanged until the partner has read.
       staging_free(lane);
-      reinterpret_cast<float2*>(stg + 4096)[lane] = make_float2(m_used, l);
+      reinterpret_cast<float*>(stg + 4096)[lane] = l;
       pair_sync(quarter);
-      const float2 oth = reinterpret_cast<const float2*>(stg + ((warp ^ 4) - warp) * 8192 + 4096)[lane];
+      const float l_oth = reinterpret_cast<const float*>(stg + ((warp ^ 4) - warp) * 8192 + 4096)[lane];
       pair_sync(quarter);
-      const float m0 = kh == 0 ? m_used : oth.x, l0 = kh == 0 ? l : oth.y;
-      const float m1 = kh == 0 ? oth.x : m_used, l1 = kh == 0 ? oth.y : l;
-      const float M = fmaxf(m0, m1);
-      const float f0 = m0 == -CUDART_INF_F ? 0.f : fast_exp2(m0 - M);
-      const float f1 = m1 == -CUDART_INF_F ? 0.f : fast_exp2(m1 - M);
       const bool has_value = rowlim > 0;  // a position that saw no key, or past the sequence: zeros
-      const float inv = has_value ? 1.f / (l0 * f0 + l1 * f1) : 0.f;
-      const float g0 = f0 * inv, g1 = f1 * inv;
+      const float inv = has_value ? 1.f / (kh == 0 ? l + l_oth : l_oth + l) : 0.f;
       const int jl = i - 1;
       if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
       if (!dead) {
         tc::fence_after_sync();
 #pragma unroll 1
         for (int c = 0; c < D / 64; ++c) {
-          uint32_t a[32], b[32];
+          uint32_t a[32];
           tc::tmem_ld32(lane_base + kTmemO + c0 + c * 32, a);
-          tc::tmem_ld32(lane_base + kTmemO + D + c0 + c * 32, b);
           tc::tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
             if (has_value)
-              v = make_float4(__uint_as_float(a[4 * e]) * g0 + __uint_as_float(b[4 * e]) * g1,
-                              __uint_as_float(a[4 * e + 1]) * g0 + __uint_as_float(b[4 * e + 1]) * g1,
-                              __uint_as_float(a[4 * e + 2]) * g0 + __uint_as_float(b[4 * e + 2]) * g1,
-                              __uint_as_float(a[4 * e + 3]) * g0 + __uint_as_float(b[4 * e + 3]) * g1);
+              v = make_float4(__uint_as_float(a[4 * e]) * inv, __uint_as_float(a[4 * e + 1]) * inv,
+                              __uint_as_float(a[4 * e + 2]) * inv, __uint_as_float(a[4 * e + 3]) * inv);
             *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + ((e ^ (lane & 7)) << 4)) = v;
           }
           store_box(&tmO, stg + c * 4096, it.h * D + c0 + c * 32, it.j0 + quarter * 32, it.b, lane);
