@@ -101,10 +101,30 @@ struct BlkCfg {
   static_assert(kNumBars * 8 <= 512, "barrier area");
 };
 
+// Division of a non-negative int below 2^31 by a fixed positive divisor d as
+// one multiply and shift (Granlund and Montgomery, "Division by invariant
+// integers using multiplication", 1994): with l = ceil(log2 d) and
+// m = ceil(2^(31+l) / d) < 2^32, n / d = (m n) >> (31 + l) for 0 <= n < 2^31.
+struct FastDiv {
+  uint32_t m, s;
+  int d;
+  __device__ __forceinline__ int div(int n) const { return (int)(((uint64_t)m * (uint32_t)n) >> s); }
+  static FastDiv make(int d) {
+    int l = 0;
+    while ((1ll << l) < d) ++l;
+    FastDiv f;
+    f.m = (uint32_t)(((1ull << (31 + l)) + (uint64_t)d - 1) / (uint64_t)d);
+    f.s = 31 + l;
+    f.d = d;
+    return f;
+  }
+};
+
 struct BlkParams {
   const int* seq_len;
   unsigned* status;
-  int B, H, Hkv, group, T, S_cap, L;
+  int B, H, Hkv, T, S_cap, L;
+  FastDiv by_L, by_H, by_group, by_npb;
   int nqt;             // position tiles per sequence
   int npb;             // tile pairs per (b, h)
   int npairs;          // B * H * npb (below 2^31)
@@ -132,8 +152,8 @@ struct Walker {
   }
   __device__ bool next(const BlkParams& p, Item& it) {
     while (pair < p.npairs) {
-      const int k = pair % p.npb;
-      const int bh = pair / p.npb;
+      const int bh = p.by_npb.div(pair);
+      const int k = pair - bh * p.npb;
       const int qa = p.nqt - 1 - k, qb = k;
       const int e0 = e;
       if (e == 0) {
@@ -143,7 +163,7 @@ struct Walker {
         pair += gridDim.x;
       }
       if (e0 == 1 && qb >= qa) continue;  // a pair of one tile (the middle of an odd count)
-      it.b = bh / p.H;
+      it.b = p.by_H.div(bh);
       it.h = bh - it.b * p.H;
       if (it.b != cb) {  // consecutive pairs mostly share the sequence: one load per change
         const int n = p.seq_len[it.b];
@@ -155,8 +175,8 @@ struct Walker {
       it.j0 = (e0 == 0 ? qa : qb) * kBM;
       if (it.j0 < n) {
         const int jl = (it.j0 + kBM < n ? it.j0 + kBM : n) - 1;
-        it.klen = p.L * (jl / p.L);
-        it.mlim = p.L * (it.j0 / p.L);
+        it.klen = p.L * p.by_L.div(jl);
+        it.mlim = p.L * p.by_L.div(it.j0);
       } else {
         it.klen = 0;
         it.mlim = 0;
@@ -312,7 +332,7 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
           first(c);
         }
       };
-      auto kv_row = [&](const Cursor& c) { return (c.it.b * p.Hkv + c.it.h / p.group) * p.S_cap + c.t * kBN; };
+      auto kv_row = [&](const Cursor& c) { return (c.it.b * p.Hkv + p.by_group.div(c.it.h)) * p.S_cap + c.t * kBN; };
       Cursor ck, cv;
       ck.w.start();
       cv.w.start();
@@ -334,6 +354,16 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
               ck.qdone = true;
               ++q_issued;
               progressed = true;
+              {  // the next item's Q into L2, an item ahead of its load
+                Walker la = ck.w;
+                Item nx;
+                while (la.next(p, nx))
+                  if (nx.nt > 0) {
+                    for (int hd = 0; hd < C::kHalves; ++hd)
+                      tc::tma_prefetch_l2_2d(&tmQ, nx.h * D + hd * 64, nx.b * p.T + nx.j0);
+                    break;
+                  }
+              }
             }
           } else if (mbar_test_wait(&bars[B_KEMPTY + ck.i % ns], ((ck.i / ns) & 1) ^ 1)) {
             const int st = ck.i % ns;
@@ -474,7 +504,7 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
       }
       const int j = it.j0 + r;
       const bool valid = j < it.n;
-      const int rowlim = valid ? p.L * (j / p.L) : 0;  // keys below it are visible to this position
+      const int rowlim = valid ? p.L * p.by_L.div(j) : 0;  // keys below it are visible to this position
       float m_used = -CUDART_INF_F, l = 0.f;
       for (int t = 0; t < it.nt; ++t, ++i) {
         const int bi = i % kSBufs;
@@ -652,11 +682,15 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   BlkParams p;
   p.seq_len = a.kv_len;
   p.status = reinterpret_cast<unsigned*>(a.ws);
-  p.B = a.B; p.H = a.H; p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.T = a.T; p.S_cap = a.S_cap; p.L = a.block_L;
+  p.B = a.B; p.H = a.H; p.Hkv = a.Hkv; p.T = a.T; p.S_cap = a.S_cap; p.L = a.block_L;
+  p.by_L = FastDiv::make(a.block_L);
+  p.by_H = FastDiv::make(a.H);
+  p.by_group = FastDiv::make(a.H / a.Hkv);
   p.nqt = (a.T + kBM - 1) / kBM;
   p.npb = (p.nqt + 1) / 2;
   if ((long long)a.B * a.H * p.npb > 0x7fffffffLL) return cudaErrorNotSupported;
   p.npairs = a.B * a.H * p.npb;
+  p.by_npb = FastDiv::make(p.npb);
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
   int G = a.max_ctas > 0 ? a.max_ctas : sm_count();

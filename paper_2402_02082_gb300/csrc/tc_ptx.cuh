@@ -159,6 +159,14 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       : "memory");
 }
 
+// Box of a 2-D tensor map at element coordinates (x, y) into L2 only.
+__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
 // Box of a 3-D tensor map at element coordinates (x, y, z) from shared memory
 // to global memory, in this thread's current bulk async-group; elements
 // outside the tensor are not written.
