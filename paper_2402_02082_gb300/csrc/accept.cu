@@ -24,6 +24,8 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kChunk = 8192;  // logits per CTA
+constexpr int kVec = kChunk / (4 * kThreads);  // float4 loads per thread, all in flight at once
+static_assert(kChunk % (4 * kThreads) == 0, "chunk of whole float4 rounds");
 
 struct AccParams {
   const int32_t* draft;
@@ -55,7 +57,7 @@ __device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsig
 __global__ void __launch_bounds__(kThreads) tree_accept_kernel(const AccParams p) {
   __shared__ unsigned long long red[kThreads / 32];
   __shared__ int last;
-  __shared__ int sa[kMaxTree];
+  __shared__ int sa[kMaxTree], sp[kMaxTree], sd[kMaxTree];
 
   const int row = blockIdx.x / p.splits;
   const int split = blockIdx.x - row * p.splits;
@@ -67,13 +69,23 @@ __global__ void __launch_bounds__(kThreads) tree_accept_kernel(const AccParams p
   unsigned long long best = 0ull;
   if ((p.V & 3) == 0) {
     const float4* v4 = reinterpret_cast<const float4*>(lg);
-    for (int j = lo / 4 + threadIdx.x; j < hi / 4; j += kThreads) {
-      const float4 x = __ldcs(v4 + j);
-      const int i0 = 4 * j;
-      best = umax64(best, argmax_key(x.x, i0));
-      best = umax64(best, argmax_key(x.y, i0 + 1));
-      best = umax64(best, argmax_key(x.z, i0 + 2));
-      best = umax64(best, argmax_key(x.w, i0 + 3));
+    const int j0 = lo / 4 + threadIdx.x, j1 = hi / 4;
+    float4 x[kVec];
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      const int j = j0 + u * kThreads;
+      x[u] = j < j1 ? __ldcs(v4 + j) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      const int j = j0 + u * kThreads;
+      if (j < j1) {
+        const int i0 = 4 * j;
+        best = umax64(best, argmax_key(x[u].x, i0));
+        best = umax64(best, argmax_key(x[u].y, i0 + 1));
+        best = umax64(best, argmax_key(x[u].z, i0 + 2));
+        best = umax64(best, argmax_key(x[u].w, i0 + 3));
+      }
     }
   } else {
     for (int j = lo + threadIdx.x; j < hi; j += kThreads) best = umax64(best, argmax_key(__ldcs(lg + j), j));
@@ -99,7 +111,11 @@ __global__ void __launch_bounds__(kThreads) tree_accept_kernel(const AccParams p
   const int n = p.n;
   const int32_t* par = p.parent + (size_t)b * n;
   const int32_t* dr = p.draft + (size_t)b * n;
-  for (int c = lane; c < n; c += 32) sa[c] = key_index(__ldcg(&p.slots[(size_t)b * n + c]));
+  for (int c = lane; c < n; c += 32) {  // the argmaxes and the tree into shared memory for the walks
+    sa[c] = key_index(__ldcg(&p.slots[(size_t)b * n + c]));
+    sp[c] = par[c];
+    sd[c] = dr[c];
+  }
   __syncwarp();
   unsigned key = 0;
   for (int c = lane; c < n; c += 32) {
@@ -107,8 +123,8 @@ __global__ void __launch_bounds__(kThreads) tree_accept_kernel(const AccParams p
     int depth = 0;
     int x = c;
     for (int step = 0; step < kMaxTree && x != 0; ++step) {
-      const int px = par[x];
-      if (px < 0 || px >= x || dr[x] != sa[px]) { ok = false; break; }
+      const int px = sp[x];
+      if (px < 0 || px >= x || sd[x] != sa[px]) { ok = false; break; }
       ++depth;
       x = px;
     }
@@ -124,7 +140,7 @@ __global__ void __launch_bounds__(kThreads) tree_accept_kernel(const AccParams p
     int x = node;
     for (int d = depth; d >= 0; --d) {
       out_path[d] = x;
-      x = d > 0 ? par[x] : -1;
+      x = d > 0 ? sp[x] : -1;
     }
     p.len[b] = depth;
     p.bonus[b] = sa[node];
