@@ -24,9 +24,9 @@
 // it waits for the completion of P.V of tile i; three buffers keep that wait
 // off the softmax's path.
 //
-// The epilogue stages O / l per warp in two 4 KB boxes of shared memory (the
-// 128-byte swizzle) and writes them with bulk tensor stores, which drain
-// while the warps go on with the next item.
+// The epilogue stages O / l in 4 KB boxes of shared memory (the 128-byte
+// swizzle) and writes them with bulk tensor stores, which drain while the
+// warps go on with the next item.
 //
 // Work item: (sequence b, query head h, tile of 128 positions).  Tile x of a
 // (b, h) sees about x + 1 key tiles, so tile x is paired with tile
@@ -34,16 +34,22 @@
 // runs pairs c, c + G, c + 2G, ... in (b, h)-major order: the CTAs that run at
 // the same time read the keys and values of a few heads, which stay in L2.
 //
-// Roles (352 threads, one CTA per SM):
-//   warps 0-7  softmax, two groups of four: warp w reads TMEM lane quarter
-//              w % 4 (one thread per position) and key half w / 4 of every
-//              tile, with packed f32x2 arithmetic; then the item's epilogue,
-//              each group writing half of the head dims.
-//   warp 8     producer: lane 0 loads the Q tile and feeds the K and V rings
-//              with 2-D TMA, polling the free slots of both.
-//   warp 9     S issue (lane 0) and the TMEM allocation.
-//   warp 10    P.V issue (lane 0).  Separate issuers keep S of later tiles
-//              from queueing behind the wait for this tile's P.
+// Roles (512 threads, one CTA per SM; setmaxnreg gives the softmax warps 168
+// registers a thread and the others 88):
+//   warps 0-7   softmax, two groups of four: warp w reads TMEM lane quarter
+//               w % 4 (one thread per position) and key half w / 4 of every
+//               tile, with packed f32x2 arithmetic; at the end of an item it
+//               hands its row sums to the epilogue warps.
+//   warp 8      producer: lane 0 loads the Q tile and feeds the K and V rings
+//               with 2-D TMA, polling the free slots of both.
+//   warp 9      S issue (lane 0) and the TMEM allocation.
+//   warp 10     P.V issue (lane 0).  Separate issuers keep S of later tiles
+//               from queueing behind the wait for this tile's P.
+//   warp 11     idle (completes the register split's warpgroup).
+//   warps 12-15 epilogue: warp 12 + q reads lane quarter q of O once the
+//               item's last P.V is done, frees O for the next item and writes
+//               O / l with bulk tensor stores, while the softmax warps are
+//               already on the next item.
 //
 // Online softmax in the log2 domain with a lazy reference max: O is rescaled
 // in TMEM only when a tile's max exceeds the reference by more than 8 (factor
@@ -70,8 +76,10 @@ constexpr int kMaxStages = 4;     // K/V ring stages (the launch picks as many a
 constexpr int kSoftWarps = 8;     // two groups of four: the key halves of every tile
 constexpr int kProdWarp = 8;
 constexpr int kSWarp = 9;
-constexpr int kPVWarp = 10;
-constexpr int kThreads = 352;
+constexpr int kPVWarp = 10;      // warp 11 only completes warpgroup 2
+constexpr int kEpiWarp0 = 12;    // warps 12-15: the item epilogues, one per TMEM lane quarter
+constexpr int kEpiWarps = 4;
+constexpr int kThreads = 512;
 constexpr int kTmemCols = 512;
 constexpr int kSBufs = 3;                   // S / P buffers at columns 0, 128, 256
 constexpr uint32_t kTmemO = kSBufs * kBN;   // the O accumulator from column 384
@@ -79,7 +87,8 @@ constexpr uint32_t kAtom = 128 * 128;       // one 128-byte-swizzle atom of 128 
 constexpr float kRescaleLog2 = 8.0f;
 
 constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
-              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_OFREE = 29, B_MDONE = 30, kNumBars = 32;
+              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_OFREE = 29, B_MDONE = 30, B_LREADY = 32, B_LFREE = 33,
+              kNumBars = 34;
 
 template <int D>
 struct BlkCfg {
@@ -87,16 +96,17 @@ struct BlkCfg {
   static constexpr uint32_t kQBytes = kHalves * kAtom;  // 128 positions x D
   static constexpr uint32_t kKV = kHalves * kAtom;      // 128 keys x D
   static constexpr uint32_t off_Q = 0;
-  // epilogue staging: per softmax warp two boxes of 32 positions x 32 fp32
-  // outputs (4 KB each, 128-byte swizzle); the second also carries the
-  // warp's (max, sum) pairs to its partner of the other key half
-  static constexpr uint32_t kStage = kSoftWarps * 2 * 4096;
+  // epilogue staging: per epilogue warp its 32 positions x D fp32 outputs as
+  // D/32 boxes of 32 x 32 (4 KB each, 128-byte swizzle)
+  static constexpr uint32_t kStage = kEpiWarps * (D / 32) * 4096;
   static constexpr uint32_t off_stg = off_Q + kQBytes;
   static constexpr uint32_t off_K = off_stg + kStage;
   static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKV; }
   static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKV; }
   static __host__ __device__ uint32_t off_misc(int ns) { return off_bar(ns) + 512; }
-  static size_t smem_bytes(int ns) { return 1024 + off_misc(ns) + 16; }
+  // the item's row sums, [key half][position], from the softmax to the epilogue warps
+  static __host__ __device__ uint32_t off_lsum(int ns) { return off_misc(ns) + 16; }
+  static size_t smem_bytes(int ns) { return 1024 + off_lsum(ns) + 2 * kBM * 4; }
   static_assert(kTmemO + D <= kTmemCols, "TMEM columns");
   static_assert(kNumBars * 8 <= 512, "barrier area");
 };
@@ -270,8 +280,16 @@ __device__ __forceinline__ void pair_sync(int quarter) {
   asm volatile("bar.sync %0, 64;" ::"r"(4 + quarter) : "memory");
 }
 
+// Warpgroup register split (setmaxnreg): the two softmax warpgroups take 168
+// registers a thread, the producer / MMA and epilogue warpgroups give theirs
+// down to 88, so that each SM sub-partition's 16384 registers hold its four
+// warps (2 x 168 + 2 x 88 = 512 per lane) -- exactly the 512 x 128 the block
+// is launched with.
+__device__ __forceinline__ void regs_up() { asm volatile("setmaxnreg.inc.sync.aligned.u32 168;" ::: "memory"); }
+__device__ __forceinline__ void regs_down() { asm volatile("setmaxnreg.dec.sync.aligned.u32 88;" ::: "memory"); }
+
 template <int D>
-__global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 16384 registers
+__global__ void __launch_bounds__(kThreads, 1)
     block_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
                       const BlkParams p) {
@@ -282,13 +300,15 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
   const uint32_t off_V = C::off_V(ns);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(ns));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
+  float* lsum = reinterpret_cast<float*>(base + C::off_lsum(ns));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int b = 0; b < kNumBars; ++b) {
-      const bool soft = (b >= B_PFULL && b < B_PFULL + kSBufs) || b == B_OFREE;
-      mbar_init(&bars[b], soft ? kSoftWarps : 1);
+      const bool soft = (b >= B_PFULL && b < B_PFULL + kSBufs) || b == B_LREADY;
+      const bool epi = b == B_OFREE || b == B_LFREE;
+      mbar_init(&bars[b], soft ? kSoftWarps : (epi ? kEpiWarps : 1));
     }
     *abort_flag = 0;
     fence_barrier_init();
@@ -301,7 +321,8 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
   __syncthreads();
   tc::fence_after_sync();
   const uint32_t tmem = *tmem_slot;
-
+  if (warp >= kSoftWarps) {
+  regs_down();
   if (warp == kProdWarp) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
@@ -475,33 +496,88 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
       tc::mma_commit(&bars[B_MDONE + role]);  // every MMA finished before TMEM is released
       mbar_drain(&bars[B_MDONE + role], 0);
     }
+  } else if (warp >= kEpiWarp0) {
+    // ------------------------------------------------------------ epilogue
+    // Warp 12 + q writes positions 32q .. 32q+31 of every item: O / (l_0 + l_1)
+    // from TMEM lane quarter q, staged in D/32 boxes and written with bulk
+    // tensor stores.  The softmax warps go on with the next item meanwhile; its
+    // first P.V waits until O has been read here.
+    const int quarter = warp - kEpiWarp0;
+    const int r = quarter * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    unsigned char* stg = base + C::off_stg + quarter * (D / 32) * 4096;
+    bool dead = false;
+    Walker w;
+    w.start();
+    Item it;
+    int i = 0, ke = 0;
+    while (w.next(p, it)) {
+      staging_free(lane);  // the previous item's stores have read the boxes
+      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + (e << 4)) = make_float4(0.f, 0.f, 0.f, 0.f);
+          store_box(&tmO, stg + c * 4096, it.h * D + c * 32, it.j0 + quarter * 32, it.b, lane);
+        }
+        continue;
+      }
+      i += it.nt;
+      const int jl = i - 1;  // the item's last tile
+      const int j = it.j0 + r;
+      // a position that saw no key, or past the sequence: zeros
+      const bool has_value = j < it.n && p.L * p.by_L.div(j) > 0;
+      if (!dead) dead = !warp_wait(&bars[B_LREADY], ke & 1, abort_flag, p.status);
+      const float l0 = lsum[r], l1 = lsum[kBM + r];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_LFREE]);
+      ++ke;
+      const float inv = has_value ? 1.f / (l0 + l1) : 0.f;
+      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+      if (!dead) {
+        tc::fence_after_sync();
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t a[32];
+          tc::tmem_ld32(lane_base + kTmemO + c * 32, a);
+          tc::tmem_wait_ld();
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (has_value)
+              v = make_float4(__uint_as_float(a[4 * q]) * inv, __uint_as_float(a[4 * q + 1]) * inv,
+                              __uint_as_float(a[4 * q + 2]) * inv, __uint_as_float(a[4 * q + 3]) * inv);
+            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + ((q ^ (lane & 7)) << 4)) = v;
+          }
+        }
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars[B_OFREE]);  // O is read: the next item's P.V may overwrite it
+      if (!dead)
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c)
+          store_box(&tmO, stg + c * 4096, it.h * D + c * 32, it.j0 + quarter * 32, it.b, lane);
+    }
+    if (lane == 0) tc::bulk_wait_all();  // the output stores have landed
+  }
   } else {
+  regs_up();
     // ------------------------------------------------------------- softmax
     const int kh = warp >> 2, quarter = warp & 3;
     const int r = quarter * 32 + lane;  // this thread's position in the tile (its TMEM lane)
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t o_col = kTmemO + kh * (D / 2);  // this group's half of the O columns
     const int sid = threadIdx.x;        // 0..255 among the softmax threads
-    const int c0 = kh * (D / 2);        // this group's half of the head dims in the output
     const float sl2 = p.scale_log2;
-    unsigned char* stg = base + C::off_stg + warp * 8192;  // this warp's two staging boxes
     bool dead = false;
     Walker w;
     w.start();
     Item it;
-    int i = 0, kq = 0;
+    int i = 0, ke = 0;  // CTA-local tile, items with keys
     while (w.next(p, it)) {
-      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros
-        staging_free(lane);
-#pragma unroll 1
-        for (int c = 0; c < D / 64; ++c) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + (e << 4)) = make_float4(0.f, 0.f, 0.f, 0.f);
-          store_box(&tmO, stg + c * 4096, it.h * D + c0 + c * 32, it.j0 + quarter * 32, it.b, lane);
-        }
-        continue;
-      }
+      if (it.nt == 0) continue;  // no visible key anywhere in the tile: the epilogue warps write zeros
       const int j = it.j0 + r;
       const bool valid = j < it.n;
       const int rowlim = valid ? p.L * p.by_L.div(j) : 0;  // keys below it are visible to this position
@@ -612,45 +688,16 @@ __global__ void __maxnreg__(168)  // 11 warps: three share a sub-partition's 163
         if (lane == 0) mbar_arrive(&bars[B_PFULL + bi]);
       }
 
-      // ---- item epilogue: group h writes head dims [h D/2, (h+1) D/2) of O / l
-      // The partner's sum (taken against the same reference max) through the
-      // second staging boxes: free again once this warp's earlier stores have
-      // read them; the second barrier keeps both unchanged until the partner has read.
-      staging_free(lane);
-      reinterpret_cast<float*>(stg + 4096)[lane] = l;
-      pair_sync(quarter);
-      const float l_oth = reinterpret_cast<const float*>(stg + ((warp ^ 4) - warp) * 8192 + 4096)[lane];
-      pair_sync(quarter);
-      const bool has_value = rowlim > 0;  // a position that saw no key, or past the sequence: zeros
-      const float inv = has_value ? 1.f / (kh == 0 ? l + l_oth : l_oth + l) : 0.f;
-      const int jl = i - 1;
-      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
-      if (!dead) {
-        tc::fence_after_sync();
-#pragma unroll 1
-        for (int c = 0; c < D / 64; ++c) {
-          uint32_t a[32];
-          tc::tmem_ld32(lane_base + kTmemO + c0 + c * 32, a);
-          tc::tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (has_value)
-              v = make_float4(__uint_as_float(a[4 * e]) * inv, __uint_as_float(a[4 * e + 1]) * inv,
-                              __uint_as_float(a[4 * e + 2]) * inv, __uint_as_float(a[4 * e + 3]) * inv);
-            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + ((e ^ (lane & 7)) << 4)) = v;
-          }
-          store_box(&tmO, stg + c * 4096, it.h * D + c0 + c * 32, it.j0 + quarter * 32, it.b, lane);
-        }
-      }
-      tc::fence_before_sync();
+      // The item's sums to the epilogue warps (the buffer is free once they
+      // have read the previous item's).
+      if (!dead) dead = !warp_wait(&bars[B_LFREE], (ke & 1) ^ 1, abort_flag, p.status);
+      lsum[kh * kBM + r] = l;
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars[B_OFREE]);
-      ++kq;
+      if (lane == 0) mbar_arrive(&bars[B_LREADY]);
+      ++ke;
     }
   }
 
-  if (warp < kSoftWarps && lane == 0) tc::bulk_wait_all();  // the output stores have landed
   __syncwarp();  // the producer and MMA warps reconverge after their single-lane loops
   tc::fence_before_sync();
   __syncthreads();
