@@ -96,17 +96,19 @@ struct BlkCfg {
   static constexpr uint32_t kQBytes = kHalves * kAtom;  // 128 positions x D
   static constexpr uint32_t kKV = kHalves * kAtom;      // 128 keys x D
   static constexpr uint32_t off_Q = 0;
-  // epilogue staging: per epilogue warp its 32 positions x D fp32 outputs as
-  // D/32 boxes of 32 x 32 (4 KB each, 128-byte swizzle)
-  static constexpr uint32_t kStage = kEpiWarps * (D / 32) * 4096;
+  // epilogue staging: per epilogue warp two boxes of 32 positions x 32 fp32
+  // outputs (4 KB each, 128-byte swizzle): the D/32 chunks go through them in
+  // rounds of two
+  static constexpr uint32_t kStage = kEpiWarps * 2 * 4096;
   static constexpr uint32_t off_stg = off_Q + kQBytes;
   static constexpr uint32_t off_K = off_stg + kStage;
-  static __host__ __device__ uint32_t off_V(int ns) { return off_K + ns * kKV; }
-  static __host__ __device__ uint32_t off_bar(int ns) { return off_V(ns) + ns * kKV; }
-  static __host__ __device__ uint32_t off_misc(int ns) { return off_bar(ns) + 512; }
+  // K ring of nk stages, then the V ring of nv
+  static __host__ __device__ uint32_t off_V(int nk) { return off_K + nk * kKV; }
+  static __host__ __device__ uint32_t off_bar(int nk, int nv) { return off_V(nk) + nv * kKV; }
+  static __host__ __device__ uint32_t off_misc(int nk, int nv) { return off_bar(nk, nv) + 512; }
   // the item's row sums, [key half][position], from the softmax to the epilogue warps
-  static __host__ __device__ uint32_t off_lsum(int ns) { return off_misc(ns) + 16; }
-  static size_t smem_bytes(int ns) { return 1024 + off_lsum(ns) + 2 * kBM * 4; }
+  static __host__ __device__ uint32_t off_lsum(int nk, int nv) { return off_misc(nk, nv) + 16; }
+  static size_t smem_bytes(int nk, int nv) { return 1024 + off_lsum(nk, nv) + 2 * kBM * 4; }
   static_assert(kTmemO + D <= kTmemCols, "TMEM columns");
   static_assert(kNumBars * 8 <= 512, "barrier area");
 };
@@ -138,7 +140,7 @@ struct BlkParams {
   int nqt;             // position tiles per sequence
   int npb;             // tile pairs per (b, h)
   int npairs;          // B * H * npb (below 2^31)
-  int ns;              // K/V stages
+  int nk, nv;          // K and V ring stages
   float scale_log2;
 };
 
@@ -296,12 +298,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   using C = BlkCfg<D>;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  const int ns = p.ns;
-  const uint32_t off_V = C::off_V(ns);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(ns));
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
-  float* lsum = reinterpret_cast<float*>(base + C::off_lsum(ns));
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
+  const int k_stages = p.nk, v_stages = p.nv;  // K and V ring depths
+  const uint32_t off_V = C::off_V(k_stages);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + C::off_bar(k_stages, v_stages));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(k_stages, v_stages));
+  float* lsum = reinterpret_cast<float*>(base + C::off_lsum(k_stages, v_stages));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(k_stages, v_stages) + 4);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -386,8 +388,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                   }
               }
             }
-          } else if (mbar_test_wait(&bars[B_KEMPTY + ck.i % ns], ((ck.i / ns) & 1) ^ 1)) {
-            const int st = ck.i % ns;
+          } else if (mbar_test_wait(&bars[B_KEMPTY + ck.i % k_stages], ((ck.i / k_stages) & 1) ^ 1)) {
+            const int st = ck.i % k_stages;
             mbar_arrive_expect_tx(&bars[B_KFULL + st], C::kKV);
             for (int hd = 0; hd < C::kHalves; ++hd)
               tc::tma_load_2d(base + C::off_K + st * C::kKV + hd * kAtom, &tmK, hd * 64, kv_row(ck),
@@ -396,8 +398,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             progressed = true;
           }
         }
-        if (cv.has && mbar_test_wait(&bars[B_VEMPTY + cv.i % ns], ((cv.i / ns) & 1) ^ 1)) {
-          const int st = cv.i % ns;
+        if (cv.has && mbar_test_wait(&bars[B_VEMPTY + cv.i % v_stages], ((cv.i / v_stages) & 1) ^ 1)) {
+          const int st = cv.i % v_stages;
           mbar_arrive_expect_tx(&bars[B_VFULL + st], C::kKV);
           for (int hd = 0; hd < C::kHalves; ++hd)
             tc::tma_load_2d(base + off_V + st * C::kKV + hd * kAtom, &tmV, hd * 64, kv_row(cv), &bars[B_VFULL + st],
@@ -424,8 +426,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (ck.has || cv.has) {  // aborted: let issued loads land before the CTA exits
-        for (int j = (ck.i > ns ? ck.i - ns : 0); j < ck.i; ++j) mbar_drain(&bars[B_KFULL + j % ns], (j / ns) & 1);
-        for (int j = (cv.i > ns ? cv.i - ns : 0); j < cv.i; ++j) mbar_drain(&bars[B_VFULL + j % ns], (j / ns) & 1);
+        for (int j = (ck.i > k_stages ? ck.i - k_stages : 0); j < ck.i; ++j)
+          mbar_drain(&bars[B_KFULL + j % k_stages], (j / k_stages) & 1);
+        for (int j = (cv.i > v_stages ? cv.i - v_stages : 0); j < cv.i; ++j)
+          mbar_drain(&bars[B_VFULL + j % v_stages], (j / v_stages) & 1);
         if (q_issued > 0) mbar_drain(&bars[B_QFULL], (q_issued - 1) & 1);
       }
     }
@@ -449,33 +453,33 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (s_role) {
             // S(i) = Q K(i)^T into buffer i % 3, once P.V of tile i - 3 has read that buffer
             if ((t == 0 && !mbar_wait(&bars[B_QFULL], kq & 1, abort_flag, p.status)) ||
-                !mbar_wait(&bars[B_KFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
+                !mbar_wait(&bars[B_KFULL + i % k_stages], (i / k_stages) & 1, abort_flag, p.status) ||
                 !mbar_wait(&bars[B_BFREE + bi], ((i / kSBufs) & 1) ^ 1, abort_flag, p.status)) {
               ok = false;
               break;
             }
             tc::fence_after_sync();
-            const uint64_t dK = tc::sw128_desc(sK + (i % ns) * C::kKV, 16, 1024);
+            const uint64_t dK = tc::sw128_desc(sK + (i % k_stages) * C::kKV, 16, 1024);
 #pragma unroll
             for (int ks = 0; ks < D / 16; ++ks) {
               const uint64_t step = desc_step((ks >> 2) * kAtom + (ks & 3) * 32);
               tc::mma_bf16(tmem + bi * kBN, dQ + step, dK + step, idS, ks > 0 ? 1u : 0u);
             }
             tc::mma_commit(&bars[B_SFULL + bi]);
-            tc::mma_commit(&bars[B_KEMPTY + i % ns]);
+            tc::mma_commit(&bars[B_KEMPTY + i % k_stages]);
             if (t == it.nt - 1) tc::mma_commit(&bars[B_QEMPTY]);
           } else {
             // O (+)= P_0(i) V_0(i) + P_1(i) V_1(i) over the key halves h = 0, 1: P_h in
             // columns 64h .. 64h+31 of buffer i % 3
             const bool first = t == 0;
             if (!mbar_wait(&bars[B_PFULL + bi], (i / kSBufs) & 1, abort_flag, p.status) ||
-                !mbar_wait(&bars[B_VFULL + i % ns], (i / ns) & 1, abort_flag, p.status) ||
+                !mbar_wait(&bars[B_VFULL + i % v_stages], (i / v_stages) & 1, abort_flag, p.status) ||
                 (first && kq > 0 && !mbar_wait(&bars[B_OFREE], (kq - 1) & 1, abort_flag, p.status))) {
               ok = false;
               break;
             }
             tc::fence_after_sync();
-            const uint64_t dV = tc::sw128_desc(sV + (i % ns) * C::kKV, kAtom, 1024);
+            const uint64_t dV = tc::sw128_desc(sV + (i % v_stages) * C::kKV, kAtom, 1024);
             const uint32_t pcol = tmem + bi * kBN;
             if (first) {
               tc::mma_bf16_ts(tmem + kTmemO, pcol, dV, idO, 0u);
@@ -485,7 +489,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int ks = 1; ks < kBN / 16; ++ks)
               tc::mma_bf16_ts(tmem + kTmemO, pcol + (ks >> 2) * 64 + (ks & 3) * 8, dV + desc_step(ks * 16 * 128), idO, 1u);
-            tc::mma_commit(&bars[B_VEMPTY + i % ns]);
+            tc::mma_commit(&bars[B_VEMPTY + i % v_stages]);
             tc::mma_commit(&bars[B_ODONE + (i & 1)]);
             tc::mma_commit(&bars[B_BFREE + bi]);
           }
@@ -505,7 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp - kEpiWarp0;
     const int r = quarter * 32 + lane;
     const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
-    unsigned char* stg = base + C::off_stg + quarter * (D / 32) * 4096;
+    unsigned char* stg = base + C::off_stg + quarter * 2 * 4096;  // this warp's two boxes
     bool dead = false;
     Walker w;
     w.start();
@@ -513,14 +517,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     int i = 0, ke = 0;
     while (w.next(p, it)) {
       staging_free(lane);  // the previous item's stores have read the boxes
-      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros
-#pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
+      if (it.nt == 0) {  // no visible key anywhere in the tile: zeros, every chunk from the first box
 #pragma unroll
-          for (int e = 0; e < 8; ++e)
-            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + (e << 4)) = make_float4(0.f, 0.f, 0.f, 0.f);
-          store_box(&tmO, stg + c * 4096, it.h * D + c * 32, it.j0 + quarter * 32, it.b, lane);
-        }
+        for (int e = 0; e < 8; ++e)
+          *reinterpret_cast<float4*>(stg + lane * 128 + (e << 4)) = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) store_box(&tmO, stg, it.h * D + c * 32, it.j0 + quarter * 32, it.b, lane);
         continue;
       }
       i += it.nt;
@@ -535,30 +537,37 @@ __global__ void __launch_bounds__(kThreads, 1)
       ++ke;
       const float inv = has_value ? 1.f / (l0 + l1) : 0.f;
       if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
-      if (!dead) {
-        tc::fence_after_sync();
+      // rounds of two chunks: read from TMEM into the two boxes, then their stores
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t a[32];
-          tc::tmem_ld32(lane_base + kTmemO + c * 32, a);
-          tc::tmem_wait_ld();
+      for (int c2 = 0; c2 < D / 32; c2 += 2) {
+        if (c2 > 0) staging_free(lane);  // the previous round's stores have read the boxes
+        if (!dead) {
+          tc::fence_after_sync();
+#pragma unroll 1
+          for (int c = c2; c < c2 + 2; ++c) {
+            uint32_t a[32];
+            tc::tmem_ld32(lane_base + kTmemO + c * 32, a);
+            tc::tmem_wait_ld();
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (has_value)
-              v = make_float4(__uint_as_float(a[4 * q]) * inv, __uint_as_float(a[4 * q + 1]) * inv,
-                              __uint_as_float(a[4 * q + 2]) * inv, __uint_as_float(a[4 * q + 3]) * inv);
-            *reinterpret_cast<float4*>(stg + c * 4096 + lane * 128 + ((q ^ (lane & 7)) << 4)) = v;
+            for (int q = 0; q < 8; ++q) {
+              float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+              if (has_value)
+                v = make_float4(__uint_as_float(a[4 * q]) * inv, __uint_as_float(a[4 * q + 1]) * inv,
+                                __uint_as_float(a[4 * q + 2]) * inv, __uint_as_float(a[4 * q + 3]) * inv);
+              *reinterpret_cast<float4*>(stg + (c - c2) * 4096 + lane * 128 + ((q ^ (lane & 7)) << 4)) = v;
+            }
           }
         }
-      }
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars[B_OFREE]);  // O is read: the next item's P.V may overwrite it
-      if (!dead)
+        if (c2 + 2 == D / 32) {  // O is read: the next item's P.V may overwrite it
+          tc::fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars[B_OFREE]);
+        }
+        if (!dead)
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c)
-          store_box(&tmO, stg + c * 4096, it.h * D + c * 32, it.j0 + quarter * 32, it.b, lane);
+          for (int c = c2; c < c2 + 2; ++c)
+            store_box(&tmO, stg + (c - c2) * 4096, it.h * D + c * 32, it.j0 + quarter * 32, it.b, lane);
+      }
     }
     if (lane == 0) tc::bulk_wait_all();  // the output stores have landed
   }
@@ -673,8 +682,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const int vrows = it.klen - t * kBN;
         if (vrows < kBN) {  // the item's last tile: clear V rows past its last visible key
-          const int st = i % ns;
-          if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (i / ns) & 1, abort_flag, p.status);
+          const int st = i % v_stages;
+          if (!dead) dead = !warp_wait(&bars[B_VFULL + st], (i / v_stages) & 1, abort_flag, p.status);
           if (!dead)
             for (int idx = sid; idx < (kBN - vrows) * C::kHalves * 8; idx += kSoftWarps * 32) {
               const int row = vrows + idx / (C::kHalves * 8), rem = idx % (C::kHalves * 8);
@@ -717,9 +726,16 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  int ns = kMaxStages;
-  while (ns > 2 && C::smem_bytes(ns) > (size_t)limit) --ns;
-  if (C::smem_bytes(ns) > (size_t)limit) return cudaErrorNotSupported;
+  // As many stages as fit, the K ring first: S runs up to three tiles ahead of
+  // P.V, so the keys are needed earlier than the values.
+  int nk = kMaxStages, nv = kMaxStages;
+  while ((nk > 2 || nv > 2) && C::smem_bytes(nk, nv) > (size_t)limit) {
+    if (nv >= nk && nv > 2)
+      --nv;
+    else
+      --nk;
+  }
+  if (C::smem_bytes(nk, nv) > (size_t)limit) return cudaErrorNotSupported;
   CUtensorMap mq, mk, mv, mo;
   const long long kv_rows = (long long)a.B * a.Hkv * a.S_cap;
   if (!make_bf16_map(&mq, a.q, (long long)a.B * a.T, (long long)a.H * D, (long long)a.H * D, kBM) ||
@@ -738,12 +754,13 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   if ((long long)a.B * a.H * p.npb > 0x7fffffffLL) return cudaErrorNotSupported;
   p.npairs = a.B * a.H * p.npb;
   p.by_npb = FastDiv::make(p.npb);
-  p.ns = ns;
+  p.nk = nk;
+  p.nv = nv;
   p.scale_log2 = a.scale * kLog2e;
   int G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > p.npairs) G = p.npairs;
   if (G < 1) G = 1;
-  block_attn_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(ns), st>>>(mq, mk, mv, mo, p);
+  block_attn_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(nk, nv), st>>>(mq, mk, mv, mo, p);
   return cudaGetLastError();
 }
 
