@@ -56,6 +56,48 @@ def test_block_cross_attn(B, T, H, H_kv, D, L, seq_len, max_ctas):
         assert_attn_close(got, want, live, f"block mask T{T} H{H}/{H_kv} L{L}")
 
 
+def _random_block_case(seed):
+    """A seeded random shape: sequences, positions, heads and their grouping,
+    head dim, block length, ragged lengths (some zero) and a forced CTA count."""
+    g = np.random.default_rng(seed)
+    D = int(g.choice([64, 128]))
+    H_kv = int(g.choice([1, 2, 4]))
+    H = H_kv * int(g.choice([1, 2, 4]))
+    B = int(g.integers(1, 4))
+    T = int(g.integers(1, 700))
+    L = int(g.choice([1, 2, 3, 5, 7, 16, 200]))
+    seq_len = [int(g.integers(0, T + 1)) if g.random() < 0.5 else T for _ in range(B)]
+    max_ctas = int(g.choice([0, 0, 1, 2, 3, 5]))
+    return B, T, H, H_kv, D, L, seq_len, max_ctas
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_block_cross_attn_random_shapes(seed):
+    """Random shapes against the oracle; every output written, the device
+    status clean (a wait that ran out would show here)."""
+    B, T, H, H_kv, D, L, seq_len, max_ctas = _random_block_case(4200 + seed)
+    S_cap = (T + 15) // 16 * 16
+    K = synth.normal_values(5000 + seed, 1, (B, H_kv, S_cap, D), "bf16")
+    V = synth.normal_values(5000 + seed, 2, (B, H_kv, S_cap, D), "bf16")
+    q = synth.normal_values(5000 + seed, 3, (B, T, H, D), "bf16")
+    desc = gb.make_desc(B, H, D, S_cap, gb.GLIDE_BF16, H_kv=H_kv)
+    ws = torch.zeros(gb.glide_block_attn_workspace_bytes(desc, T), dtype=torch.uint8, device="cuda")
+    out = torch.full((B, T, H, D), float("nan"), device="cuda")
+    gb.glide_block_cross_attn(dev(q), dev(K), dev(V), dev(np.asarray(seq_len, np.int32)), L, out, ws,
+                              max_ctas=max_ctas)
+    torch.cuda.synchronize()
+    assert gb.glide_read_device_status(ws) == gb.GLIDE_OK
+    got = out.cpu().numpy()
+    assert np.isfinite(got).all(), "every output element is written"
+    want = oracle.block_cross_attn(q, K, V, seq_len, L)
+    for b, n in enumerate(seq_len):
+        dead = [j for j in range(T) if j < L or j >= n]
+        assert np.all(got[b, dead] == 0.0)
+    live = [(b, h) for b in range(B) for h in range(H) if seq_len[b] > L]
+    if live:
+        assert_attn_close(got, want, live, f"block mask random case {seed}")
+
+
 def test_block_cross_attn_rising_scores():
     """Keys whose norm grows along the sequence push each key tile's maximum
     score far above the previous ones, so the lazy reference max moves and O
