@@ -13,7 +13,8 @@
 // buffers of 128 columns and the O accumulator (D columns).  Two softmax
 // groups take the two 64-key halves of every tile, so every SM sub-partition
 // runs two softmax warps and one warp's loads, maxima and stores overlap the
-// other's exponentials (the MUFU unit is the softmax's bound).  The partners
+// other's exponentials (the softmax is latency-bound: at 32 exponentials per
+// clock per SM the MUFU unit is busy about a third of a tile).  The partners
 // of a lane quarter agree on each tile's row max through one TMEM column of
 // their halves, so both halves share one reference max and accumulate into
 // the one O; each group rescales, and at the end writes, its half of O's
@@ -24,9 +25,11 @@
 // it waits for the completion of P.V of tile i; three buffers keep that wait
 // off the softmax's path.
 //
-// The epilogue stages O / l in 4 KB boxes of shared memory (the 128-byte
-// swizzle) and writes them with bulk tensor stores, which drain while the
-// warps go on with the next item.
+// The K and V rings have separate depths, the keys' deeper (S runs up to
+// three tiles ahead of P.V): 3 and 2 stages of 32 KB for D = 128, what the
+// shared memory holds next to Q and the epilogue staging.  The epilogue stages
+// O / l in 4 KB boxes of shared memory (the 128-byte swizzle) and writes them
+// with bulk tensor stores, which drain while the warps go on.
 //
 // Work item: (sequence b, query head h, tile of 128 positions).  Tile x of a
 // (b, h) sees about x + 1 key tiles, so tile x is paired with tile
