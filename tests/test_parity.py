@@ -115,6 +115,44 @@ def test_tree_sizes(n, dtype, D):
     assert c.workspaces_clean()
 
 
+def _random_attn_case(seed):
+    """A seeded random shape: batch, heads, head dim, dtype, ragged cache
+    lengths (some zero), tree size and shape, and a forced CTA count."""
+    g = np.random.default_rng(seed)
+    B = int(g.integers(1, 6))
+    H = int(g.integers(1, 9))
+    D = int(g.choice([64, 128]))
+    dtype = str(g.choice(["bf16", "bf16", "f32"]))
+    kv = [int(g.integers(0, 700)) if g.random() < 0.8 else 0 for _ in range(B)]
+    if max(kv) == 0:
+        kv[0] = 1
+    n = int(g.choice([1, 2, 6, 17, 40, 64]))
+    tree = str(g.choice(["random", "chain"]))
+    max_ctas = int(g.choice([0, 0, 1, 3, 11, 1000]))
+    return B, H, D, dtype, kv, n, tree, max_ctas
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_random_shapes(seed):
+    """Cross-attention and tree verification of random shapes against the
+    oracle, with the workspace left clean (no wait ran out, counters re-armed)."""
+    B, H, D, dtype, kv, n, tree, max_ctas = _random_attn_case(6100 + seed)
+    c = small_case(B, H, D, dtype, kv, n, seed=6100 + seed, tree=tree)
+    live = [(b, h) for b in range(B) for h in range(H) if kv[b] > 0]
+    got = c.cross(max_ctas=max_ctas)
+    want = oracle.cross_attn(c.case["q_draft"][0], c.case["K"], c.case["V"], kv)
+    for b in range(B):
+        if kv[b] == 0:
+            assert np.array_equal(got[b], np.zeros_like(got[b]))
+    if live:
+        assert_attn_close(got, want, live, f"cross random case {seed}")
+    want = oracle.tree_verify_attn(c.case["q_tree"], c.case["parent_idx"], c.case["K"], c.case["V"], kv)
+    for flags in (0, gb.GLIDE_FLAG_FORCE_FMA):
+        assert_attn_close(c.tree(flags=flags, max_ctas=max_ctas), want, None,
+                          f"tree random case {seed} flags={flags}")
+    assert c.workspaces_clean()
+
+
 def test_tree_chain_and_forest():
     c = small_case(2, 2, 128, "bf16", [70, 3], 9, seed=41, tree="chain")
     want = oracle.tree_verify_attn(c.case["q_tree"], c.case["parent_idx"], c.case["K"], c.case["V"], [70, 3])
