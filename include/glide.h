@@ -285,9 +285,10 @@ size_t glide_block_attn_workspace_bytes(const glide_attn_desc* desc, int32_t T);
  * q [B,T,H,D] bf16; K_cache/V_cache [B,H_kv,S_cap,D] bf16 holding the target's
  * keys/values of positions 0..T-1; seq_len [B] int32 on the device (clamped to
  * [0,T]); out [B,T,H,D] fp32, every element written (no pre-zeroing needed).
- * 1 <= T <= S_cap, L >= 1.  fp32 inputs, or B*T or B*H_kv*S_cap beyond 2^31 - 128
- * rows (32-bit TMA coordinates): GLIDE_ERR_UNSUPPORTED.  The workspace holds only
- * the device status word (glide_block_attn_workspace_bytes).
+ * 1 <= T <= S_cap, L >= 1.  fp32 inputs, B*T or B*H_kv*S_cap beyond 2^31 - 128
+ * rows (32-bit TMA coordinates), or B*H*ceil(T/256) position-tile pairs plus the
+ * CTA count beyond 2^31 - 1: GLIDE_ERR_UNSUPPORTED.  The workspace holds only the
+ * device status word (glide_block_attn_workspace_bytes).
  */
 glide_status glide_block_cross_attn(const glide_attn_desc* desc, const void* q, int32_t T, int32_t L,
                                     const void* K_cache, const void* V_cache, const int32_t* seq_len,

@@ -763,6 +763,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   int G = a.max_ctas > 0 ? a.max_ctas : sm_count();
   if (G > p.npairs) G = p.npairs;
   if (G < 1) G = 1;
+  if ((long long)p.npairs + G > 0x7fffffffLL) return cudaErrorNotSupported;  // a CTA's pair index steps by G
   block_attn_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(nk, nv), st>>>(mq, mk, mv, mo, p);
   return cudaGetLastError();
 }
