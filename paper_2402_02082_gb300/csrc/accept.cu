@@ -2,17 +2,29 @@
 // the token tree of CaPE's verification, Section 3.2).
 //
 // One launch does both steps:
-// 1. argmax over the vocabulary of every (sequence, node) logits row.  The
-//    row is cut into chunks, one CTA per chunk; a CTA reduces its chunk to one
-//    64-bit key (order-preserving float bits above the complemented index, so
-//    that the larger key is the larger value and, among equal values, the
-//    lower index) and folds it into the row's slot with atomicMax.  The scan
-//    is a plain HBM stream of the logits.
-// 2. the CTA that completes a sequence's count (atomic counter, no waiting)
-//    walks that sequence's tree with one warp: a node is accepted iff every
-//    edge on its root path matches (draft token == parent's argmax); the
-//    deepest accepted node, lowest index among equals, gives the path, its
-//    length and the bonus token.  It then re-arms the slots and the counter.
+// 1. argmax over the vocabulary of every (sequence, node) logits row, lowest
+//    index among equal maxima.  Rows are cut into chunks of kChunk logits and
+//    the chunks are dealt round-robin over a persistent grid (one CTA per SM):
+//    CTA c takes chunks c, c + G, c + 2G, ...  A producer thread streams a
+//    CTA's chunks with 1-D bulk copies (TMA) into a ring of kNS shared-memory
+//    stages, so nearly all of the logits are in flight at once; stage s always
+//    serves consumer warp s, which reduces the whole chunk (a float max over
+//    each lane's float4 groups, the index recovered from the winning group,
+//    then a warp reduction) and folds one 64-bit key (order-preserving float
+//    bits above the complemented index) into the row's slot with atomicMax.
+//    The logits are a plain HBM stream.
+// 2. every chunk is counted into its sequence's counter (release fence,
+//    atomic; nothing waits).  The warp that completes a sequence's count walks
+//    that tree: a node is accepted iff every edge on its root path matches
+//    (draft token == parent's argmax); the deepest accepted node, lowest index
+//    among equals, gives the path, its length and the bonus token.  The walk
+//    is pointer jumping over the parent array in registers (two nodes per
+//    lane, six shuffle rounds for up to 64 nodes), which gives every node its
+//    acceptance, depth and ancestor set at once.  The warp then re-arms the
+//    slots and the counter.
+// Because the chunk order is sequence-major and every CTA walks it in that
+// order, sequence b's chunks are all read before sequence b + 1's: the walks
+// of the early sequences run while the later ones still stream.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -22,10 +34,15 @@
 namespace glide {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kChunk = 8192;  // logits per CTA
-constexpr int kVec = kChunk / (4 * kThreads);  // float4 loads per thread, all in flight at once
-static_assert(kChunk % (4 * kThreads) == 0, "chunk of whole float4 rounds");
+constexpr int kNW = 12;                       // consumer warps
+constexpr int kThreads = (kNW + 1) * 32;      // + one producer warp
+constexpr int kChunk = 4096;                  // logits per chunk (16 KB)
+constexpr int kNS = kNW;                      // ring stages: stage s serves consumer warp s only
+constexpr int kGroups = kChunk / (4 * 32);    // float4 groups of a lane in a whole chunk
+constexpr size_t kRingBytes = (size_t)kNS * kChunk * sizeof(float);
+constexpr size_t kSmemBytes = kRingBytes + 2 * kNS * sizeof(uint64_t) + 16;
+static_assert(kNS % kNW == 0, "a stage must always serve the same consumer warp");
+static_assert(kMaxTree <= 64, "two tree nodes per lane");
 
 struct AccParams {
   const int32_t* draft;
@@ -38,6 +55,8 @@ struct AccParams {
   unsigned* counters;
   unsigned long long* slots;
   int B, n, V, splits;
+  long long nchunks;  // B * n * splits
+  int bulk;           // 1: rows start 16-byte aligned, chunks arrive by bulk copy; 0: consumers read global memory
 };
 
 __device__ __forceinline__ unsigned long long argmax_key(float f, int idx) {
@@ -50,103 +69,261 @@ __device__ __forceinline__ int key_index(unsigned long long k) {
   return (int)(0xffffffffu - (uint32_t)(k & 0xffffffffull));
 }
 
-__device__ __forceinline__ unsigned long long umax64(unsigned long long a, unsigned long long b) {
-  return a > b ? a : b;
+// (value, index) pairs: the larger value wins, the lower index among equals.
+__device__ __forceinline__ void warp_argmax(float& m, int& idx) {
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, m, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
+    if (om > m || (om == m && oi < idx)) {
+      m = om;
+      idx = oi;
+    }
+  }
 }
 
-__global__ void __launch_bounds__(kThreads) tree_accept_kernel(const AccParams p) {
-  __shared__ unsigned long long red[kThreads / 32];
-  __shared__ int last;
-  __shared__ int sa[kMaxTree], sp[kMaxTree], sd[kMaxTree];
+// Value of node `c`'s copy of a per-node quantity held two nodes per lane
+// (v0 for node lane, v1 for node lane + 32).  All lanes must call.
+__device__ __forceinline__ uint32_t gather(uint32_t v0, uint32_t v1, int c) {
+  const uint32_t x0 = __shfl_sync(0xffffffffu, v0, c & 31);
+  const uint32_t x1 = __shfl_sync(0xffffffffu, v1, c & 31);
+  return c >= 32 ? x1 : x0;
+}
 
-  const int row = blockIdx.x / p.splits;
-  const int split = blockIdx.x - row * p.splits;
-  const int b = row / p.n;
-  const float* lg = p.logits + (size_t)row * p.V;
-  const int lo = split * kChunk;
-  const int hi = min(p.V, lo + kChunk);
+// Per-node state of the walk, packed: bit 16 = every edge of the covered part
+// of the root path matches, bits 8..15 = edges covered, bits 0..7 = the next
+// ancestor still to cover + 1 (0: the root has been reached).
+__device__ __forceinline__ uint32_t pack(bool ok, int d, int p) {
+  return (ok ? 0x10000u : 0u) | ((uint32_t)d << 8) | (uint32_t)(p + 1);
+}
 
-  unsigned long long best = 0ull;
-  if ((p.V & 3) == 0) {
-    const float4* v4 = reinterpret_cast<const float4*>(lg);
-    const int j0 = lo / 4 + threadIdx.x, j1 = hi / 4;
-    float4 x[kVec];
-#pragma unroll
-    for (int u = 0; u < kVec; ++u) {
-      const int j = j0 + u * kThreads;
-      x[u] = j < j1 ? __ldcs(v4 + j) : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll
-    for (int u = 0; u < kVec; ++u) {
-      const int j = j0 + u * kThreads;
-      if (j < j1) {
-        const int i0 = 4 * j;
-        best = umax64(best, argmax_key(x[u].x, i0));
-        best = umax64(best, argmax_key(x[u].y, i0 + 1));
-        best = umax64(best, argmax_key(x[u].z, i0 + 2));
-        best = umax64(best, argmax_key(x[u].w, i0 + 3));
-      }
-    }
-  } else {
-    for (int j = lo + threadIdx.x; j < hi; j += kThreads) best = umax64(best, argmax_key(__ldcs(lg + j), j));
-  }
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, off));
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) red[warp] = best;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    unsigned long long k = red[0];
-    for (int w = 1; w < kThreads / 32; ++w) k = umax64(k, red[w]);
-    atomicMax(&p.slots[row], k);
-    __threadfence();
-    const unsigned prev = atomicAdd(&p.counters[b], 1u);
-    last = (prev == (unsigned)(p.splits * p.n - 1)) ? 1 : 0;
-  }
-  __syncthreads();
-  if (!last || warp != 0) return;
-
-  // ---- tree walk for sequence b (one warp)
-  __threadfence();
+// Walks sequence b's tree (one whole warp; every chunk of b has been counted).
+__device__ void walk_tree(const AccParams& p, int b, int lane) {
+  __threadfence();  // the other chunks' slot updates were fenced before their counts
   const int n = p.n;
-  const int32_t* par = p.parent + (size_t)b * n;
-  const int32_t* dr = p.draft + (size_t)b * n;
-  for (int c = lane; c < n; c += 32) {  // the argmaxes and the tree into shared memory for the walks
-    sa[c] = key_index(__ldcg(&p.slots[(size_t)b * n + c]));
-    sp[c] = par[c];
-    sd[c] = dr[c];
-  }
-  __syncwarp();
-  unsigned key = 0;
-  for (int c = lane; c < n; c += 32) {
-    bool ok = true;
-    int depth = 0;
-    int x = c;
-    for (int step = 0; step < kMaxTree && x != 0; ++step) {
-      const int px = sp[x];
-      if (px < 0 || px >= x || sd[x] != sa[px]) { ok = false; break; }
-      ++depth;
-      x = px;
-    }
-    if (ok) key = max(key, ((unsigned)depth << 8) | (unsigned)(255 - c));
-  }
+  const size_t base = (size_t)b * n;
+  const int c0 = lane, c1 = lane + 32;
+  const bool h0 = c0 < n, h1 = c1 < n;
+  const unsigned long long s0 = h0 ? __ldcg(&p.slots[base + c0]) : 0ull;
+  const unsigned long long s1 = h1 ? __ldcg(&p.slots[base + c1]) : 0ull;
+  const int par0 = h0 ? p.parent[base + c0] : -1, par1 = h1 ? p.parent[base + c1] : -1;
+  const int dr0 = h0 ? p.draft[base + c0] : 0, dr1 = h1 ? p.draft[base + c1] : 0;
+  const int a0 = key_index(s0), a1 = key_index(s1);  // argmax of each node's row
+
+  // An edge matches when the node's draft token is its parent's argmax; a
+  // parent outside [0, c) leaves the node unreachable.  The root always holds.
+  const bool v0 = par0 >= 0 && par0 < c0, v1 = par1 >= 0 && par1 < c1;
+  const int pa0 = (int)gather((uint32_t)a0, (uint32_t)a1, v0 ? par0 : 0);
+  const int pa1 = (int)gather((uint32_t)a0, (uint32_t)a1, v1 ? par1 : 0);
+  const bool ok0 = h0 && (c0 == 0 || (v0 && dr0 == pa0));
+  const bool ok1 = h1 && v1 && dr1 == pa1;
+  const int p0 = (c0 > 0 && ok0) ? par0 : -1, p1 = ok1 ? par1 : -1;
+  uint32_t w0 = pack(ok0, p0 >= 0 ? 1 : 0, p0), w1 = pack(ok1, p1 >= 0 ? 1 : 0, p1);
+  // ancestor-or-self sets (64-bit, low and high words)
+  uint32_t m0l = h0 ? (1u << c0) : 0u, m0h = 0u;
+  uint32_t m1l = 0u, m1h = h1 ? (1u << (c1 - 32)) : 0u;
+
+  // Pointer jumping: each round doubles the covered part of every root path
+  // (all lanes read the previous round's values); 2^6 = 64 > any depth.
 #pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) key = max(key, __shfl_xor_sync(0xffffffffu, key, off));
+  for (int r = 0; r < 6; ++r) {
+    const int q0 = (int)(w0 & 0xffu) - 1, q1 = (int)(w1 & 0xffu) - 1;
+    const int i0 = q0 < 0 ? 0 : q0, i1 = q1 < 0 ? 0 : q1;
+    const uint32_t g0 = gather(w0, w1, i0), g1 = gather(w0, w1, i1);
+    const uint32_t gl0 = gather(m0l, m1l, i0), gh0 = gather(m0h, m1h, i0);
+    const uint32_t gl1 = gather(m0l, m1l, i1), gh1 = gather(m0h, m1h, i1);
+    if (q0 >= 0) {
+      w0 = pack((w0 & 0x10000u) && (g0 & 0x10000u), (int)((w0 >> 8) & 0xffu) + (int)((g0 >> 8) & 0xffu),
+                (int)(g0 & 0xffu) - 1);
+      m0l |= gl0;
+      m0h |= gh0;
+    }
+    if (q1 >= 0) {
+      w1 = pack((w1 & 0x10000u) && (g1 & 0x10000u), (int)((w1 >> 8) & 0xffu) + (int)((g1 >> 8) & 0xffu),
+                (int)(g1 & 0xffu) - 1);
+      m1l |= gl1;
+      m1h |= gh1;
+    }
+  }
+  const int d0 = (int)((w0 >> 8) & 0xffu), d1 = (int)((w1 >> 8) & 0xffu);
+  // deepest accepted node, lowest index among equals (the root always qualifies)
+  const unsigned k0 = (w0 & 0x10000u) ? ((unsigned)d0 << 8) | (unsigned)(255 - c0) : 0u;
+  const unsigned k1 = (w1 & 0x10000u) ? ((unsigned)d1 << 8) | (unsigned)(255 - c1) : 0u;
+  const unsigned key = __reduce_max_sync(0xffffffffu, k0 > k1 ? k0 : k1);
   const int node = 255 - (int)(key & 255u);
   const int depth = (int)(key >> 8);
-  int32_t* out_path = p.path + (size_t)b * n;
-  for (int d = depth + 1 + lane; d < n; d += 32) out_path[d] = -1;
+  const uint32_t nl = gather(m0l, m1l, node), nh = gather(m0h, m1h, node);
+  const int bonus = (int)gather((uint32_t)a0, (uint32_t)a1, node);
+
+  // The path: node c of the chosen node's ancestor set sits at position depth(c).
+  int32_t* out = p.path + base;
+  if (h0 && ((nl >> c0) & 1u)) out[d0] = c0;
+  if (h1 && ((nh >> (c1 - 32)) & 1u)) out[d1] = c1;
+  if (h0 && c0 > depth) out[c0] = -1;
+  if (h1 && c1 > depth) out[c1] = -1;
   if (lane == 0) {
-    int x = node;
-    for (int d = depth; d >= 0; --d) {
-      out_path[d] = x;
-      x = d > 0 ? sp[x] : -1;
-    }
     p.len[b] = depth;
-    p.bonus[b] = sa[node];
+    p.bonus[b] = bonus;
+    p.counters[b] = 0u;
   }
-  for (int c = lane; c < n; c += 32) p.slots[(size_t)b * n + c] = 0ull;
-  if (lane == 0) p.counters[b] = 0u;
+  if (h0) p.slots[base + c0] = 0ull;
+  if (h1) p.slots[base + c1] = 0ull;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParams p) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  float* ring = reinterpret_cast<float*>(smem);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kRingBytes);
+  uint64_t* empty = full + kNS;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(empty + kNS);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kNS; ++s) {
+      mbar_init(&full[s], 1);   // the producer's expect-tx arrival
+      mbar_init(&empty[s], 1);  // the consumer warp's release
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  // Launched as a programmatic dependent: the inputs may come from the kernel
+  // before this one, so nothing is read until that kernel has completed.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  const long long G = gridDim.x, c = blockIdx.x;
+  if (warp == kNW) {
+    // ------------------------------------------------------------ producer
+    // Lanes 1..31 put the trees into L2 for the walks; lane 0 streams chunks.
+    if (lane > 0) {
+      const long long lines = ((long long)p.B * p.n * 4 + 127) / 128;
+      for (long long l = c * 31 + (lane - 1); l < lines; l += G * 31) {
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<const char*>(p.parent) + l * 128));
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<const char*>(p.draft) + l * 128));
+      }
+      return;
+    }
+    if (!p.bulk) return;
+    const uint64_t pol = policy_evict_first();
+    long long issued = 0;
+    bool ok = true;
+    for (long long k = c; k < p.nchunks; k += G, ++issued) {
+      const int s = (int)(issued % kNS);
+      const uint32_t use = (uint32_t)(issued / kNS);
+      if (!mbar_wait(&empty[s], (use & 1u) ^ 1u, abort_flag, p.status)) { ok = false; break; }
+      const long long row = k / p.splits;
+      const int lo = (int)(k - row * p.splits) * kChunk;
+      const int cnt = min(kChunk, p.V - lo);
+      const uint32_t bytes = (uint32_t)cnt * 4u;
+      mbar_arrive_expect_tx(&full[s], bytes);
+      bulk_g2s(ring + (size_t)s * kChunk, p.logits + (size_t)row * p.V + lo, bytes, &full[s], pol);
+    }
+    if (!ok)  // let copies already issued land before the CTA exits
+      for (long long j = (issued > kNS ? issued - kNS : 0); j < issued; ++j)
+        mbar_drain(&full[j % kNS], (uint32_t)(j / kNS) & 1u);
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  // A warp folds each chunk's key into its row slot at once but counts its
+  // chunks in later, in batches of up to 32 (one lane per chunk): one fence
+  // and one round of parallel atomics per batch instead of a fence and an
+  // atomic round trip per chunk.
+  const unsigned per_seq = (unsigned)(p.n * p.splits);
+  int pend_seq = 0, npend = 0;  // lane i: the sequence of the warp's i-th uncounted chunk
+  auto count_in = [&]() {
+    __syncwarp();
+    __threadfence();  // the warp's slot updates are visible before any of its counts
+    const bool mine = lane < npend;
+    unsigned prev = 0;
+    if (mine) prev = atomicAdd(&p.counters[pend_seq], 1u);
+    unsigned done = __ballot_sync(0xffffffffu, mine && prev == per_seq - 1);
+    while (done) {  // sequences this batch completed: walk each with the whole warp
+      const int l = __ffs(done) - 1;
+      done &= done - 1;
+      walk_tree(p, __shfl_sync(0xffffffffu, pend_seq, l), lane);
+    }
+    npend = 0;
+  };
+  long long use = 0;  // chunks this warp has taken from its stage
+  for (long long j = warp; c + j * G < p.nchunks; j += kNW, ++use) {
+    const long long k = c + j * G;
+    const long long row = k / p.splits;
+    const int lo = (int)(k - row * p.splits) * kChunk;
+    const int cnt = min(kChunk, p.V - lo);
+    float m = -__int_as_float(0x7f800000);  // -inf
+    int idx = 0x7fffffff;                   // a lane that holds no logit never wins
+    if (p.bulk) {
+      if (!mbar_wait(&full[warp], (uint32_t)(use & 1), abort_flag, p.status)) break;
+      const float4* s4 = reinterpret_cast<const float4*>(ring + (size_t)warp * kChunk);
+      const int n4 = cnt >> 2;  // cnt is a multiple of 4 in this mode
+      // The lane's float4 groups in increasing index order, even and odd groups
+      // in two independent chains; a strict comparison keeps the first group
+      // holding each chain's maximum, and the index inside it comes after.
+      float ma = m, mb = m;
+      int ga = -1, gb = -1;
+      if (lane < n4) {
+        const float4 v = s4[lane];
+        ma = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
+        ga = 0;
+      }
+      if (lane + 32 < n4) {
+        const float4 v = s4[lane + 32];
+        mb = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
+        gb = 1;
+      }
+#pragma unroll 4
+      for (int i = 2; i < kGroups; i += 2) {
+        const int q = lane + 32 * i;
+        if (q < n4) {
+          const float4 v = s4[q];
+          const float g = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
+          if (g > ma) {
+            ma = g;
+            ga = i;
+          }
+        }
+        if (q + 32 < n4) {
+          const float4 v = s4[q + 32];
+          const float g = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
+          if (g > mb) {
+            mb = g;
+            gb = i + 1;
+          }
+        }
+      }
+      if (gb >= 0 && (mb > ma || (mb == ma && gb < ga))) {
+        ma = mb;
+        ga = gb;
+      }
+      if (ga >= 0) {
+        const float4 v = s4[lane + 32 * ga];
+        const int e = v.x == ma ? 0 : (v.y == ma ? 1 : (v.z == ma ? 2 : 3));
+        m = ma;
+        idx = lo + 4 * (lane + 32 * ga) + e;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[warp]);
+    } else {
+      const float* src = p.logits + (size_t)row * p.V + lo;
+      if (lane < cnt) {
+        m = __ldcs(src + lane);
+        idx = lo + lane;
+        for (int q = lane + 32; q < cnt; q += 32) {
+          const float x = __ldcs(src + q);
+          if (x > m) {
+            m = x;
+            idx = lo + q;
+          }
+        }
+      }
+    }
+    warp_argmax(m, idx);
+    if (lane == 0) atomicMax(&p.slots[row], argmax_key(m, idx));
+    if (lane == npend) pend_seq = (int)(row / p.n);
+    if (++npend == 32) count_in();
+  }
+  if (npend > 0) count_in();
 }
 
 size_t counters_bytes(int B) { return ((size_t)B * sizeof(unsigned) + 255) & ~size_t(255); }
@@ -158,6 +335,15 @@ size_t accept_workspace_bytes(int B, int n) {
 }
 
 cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st) {
+  static int configured_dev = -1;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (configured_dev != dev) {
+    e = cudaFuncSetAttribute(tree_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    configured_dev = dev;
+  }
   AccParams p;
   p.draft = a.draft; p.parent = a.parent; p.logits = a.logits;
   p.path = a.path; p.len = a.len; p.bonus = a.bonus;
@@ -167,10 +353,22 @@ cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st) {
   p.slots = reinterpret_cast<unsigned long long*>(ws + 256 + counters_bytes(a.B));
   p.B = a.B; p.n = a.n; p.V = a.V;
   p.splits = (a.V + kChunk - 1) / kChunk;
-  const long long grid = (long long)a.B * a.n * p.splits;
-  if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
-  tree_accept_kernel<<<(unsigned)grid, kThreads, 0, st>>>(p);
-  return cudaGetLastError();
+  p.nchunks = (long long)a.B * a.n * p.splits;
+  p.bulk = ((a.V & 3) == 0 && (reinterpret_cast<uintptr_t>(a.logits) & 15u) == 0) ? 1 : 0;
+  if ((long long)a.n * p.splits > 0x7fffffffLL) return cudaErrorInvalidValue;
+  long long G = sm_count();
+  if (G > p.nchunks) G = p.nchunks;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)G);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tree_accept_kernel, p);
 }
 
 }  // namespace glide

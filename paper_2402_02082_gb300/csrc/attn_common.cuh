@@ -365,13 +365,4 @@ __device__ inline void combine_partials(const Segment& s, int H, int nq, int D, 
   __syncthreads();
 }
 
-// Waits on the phase of `bar` with `parity`, bounded by time only (used to
-// drain copies still in flight after an abort).
-__device__ inline void mbar_drain(uint64_t* bar, uint32_t parity) {
-  const uint64_t t0 = global_timer_ns();
-  while (!mbar_try_wait(bar, parity)) {
-    if (global_timer_ns() - t0 > kWaitLimitNs) return;
-  }
-}
-
 }  // namespace glide

@@ -122,6 +122,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// Waits on the phase of `bar` with `parity`, bounded by time only (used to
+// drain copies still in flight after an abort).
+__device__ inline void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > kWaitLimitNs) return;
+  }
+}
+
 // ------------------------------------------------------------- bulk copies
 // 1-D bulk copy global -> this CTA's shared memory, completing `bytes` of
 // transaction count on `bar`.  dst, src and bytes must be multiples of 16.
