@@ -307,17 +307,41 @@ glide_status glide_block_cross_attn(const glide_attn_desc* desc, const void* q, 
  * - Shapes whose workspace (glide_attn_workspace_bytes(desc, 1)) exceeds
  *   32 MiB are rejected with GLIDE_ERR_UNSUPPORTED (B*H up to 7035 for D = 128,
  *   14835 for D = 64).
- * - The first call on each device looks up the array's device address; make
- *   that first call before any stream capture.
- * - Every call first clears the words that must start at zero, then reuses the
- *   array, so calls that overlap on the GPU (other streams, other host threads
- *   without ordering) race on it: serialize them.
+ * - Every call looks up the array's device address in the current device's
+ *   context (so a context created again after cudaDeviceReset is served
+ *   correctly); the first call on a device also loads the library's device
+ *   code there, so make that first call before any stream capture.  `stream`
+ *   must belong to the current device.
+ * - Every call first clears the counters that must start at zero, then reuses
+ *   the array, so calls that overlap on the GPU (other streams, other host
+ *   threads without ordering) race on it: serialize them.
+ * - A bounded wait that ran out (GLIDE_ERR_DEVICE_TIMEOUT) is recorded in the
+ *   array's status word, which calls do not clear: read it with
+ *   glide_noalloc_read_device_status.
  * - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
  */
 glide_status glide_cross_attn_noalloc(const glide_attn_desc* desc, const void* q_draft,
                                       const void* K_cache, const void* V_cache,
                                       const int32_t* kv_len, int32_t max_kv_len, float* out,
                                       glide_stream_t stream);
+
+/*
+ * The device status of glide_cross_attn_noalloc (no counterpart in the paper):
+ * waits for `stream`, then returns the status recorded in the fixed array of
+ * the current device since it was last read (GLIDE_OK or
+ * GLIDE_ERR_DEVICE_TIMEOUT) and clears it, as glide_read_device_status does for
+ * a caller's workspace.  Allocates nothing.
+ */
+glide_status glide_noalloc_read_device_status(glide_stream_t stream);
+
+/*
+ * Device address of the fixed array of glide_cross_attn_noalloc on the current
+ * device (no counterpart in the paper), for diagnostics: e.g. to point
+ * glide_selftest_wait_timeout at it.  The contents belong to the library.
+ * Returns GLIDE_ERR_INVALID for a null pointer, GLIDE_ERR_CUDA if the lookup
+ * fails.  Allocates nothing.
+ */
+glide_status glide_noalloc_scratch(void** device_ptr);
 
 /*
  * Host-side check of a parent array (HOST memory, [B,n]): every entry is -1 or

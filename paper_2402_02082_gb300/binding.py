@@ -55,6 +55,8 @@ _SIG = {
     "glide_cross_attn_noalloc": (ctypes.c_int, [ctypes.POINTER(AttnDesc), _P, _P, _P, _P, ctypes.c_int32, _P, _P]),
     "glide_validate_tree": (ctypes.c_int, [_P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
     "glide_read_device_status": (ctypes.c_int, [_P, _P]),
+    "glide_noalloc_read_device_status": (ctypes.c_int, [_P]),
+    "glide_noalloc_scratch": (ctypes.c_int, [ctypes.POINTER(ctypes.c_void_p)]),
     "glide_selftest_wait_timeout": (ctypes.c_int, [_P, ctypes.c_uint32, _P]),
     "glide_cape_workspace_bytes": (ctypes.c_size_t, [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]),
     "cape_expand": (ctypes.c_int, [_P, _P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
@@ -328,3 +330,15 @@ def glide_read_device_status(workspace: torch.Tensor, stream=None) -> int:
 def glide_selftest_wait_timeout(workspace: torch.Tensor, limit_us: int, stream=None) -> int:
     """Launch the bounded-wait self-test kernel (see include/glide.h); returns the launch status."""
     return int(lib().glide_selftest_wait_timeout(workspace.data_ptr(), int(limit_us), _stream(stream)))
+
+
+def glide_noalloc_read_device_status(stream=None) -> int:
+    """Status recorded in glide_cross_attn_noalloc's fixed array since it was last read (then cleared)."""
+    return int(lib().glide_noalloc_read_device_status(_stream(stream)))
+
+
+def glide_noalloc_scratch() -> int:
+    """Device address of glide_cross_attn_noalloc's fixed array on the current device."""
+    p = ctypes.c_void_p()
+    _check(lib().glide_noalloc_scratch(ctypes.byref(p)), "glide_noalloc_scratch")
+    return int(p.value)

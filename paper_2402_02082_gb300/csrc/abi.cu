@@ -99,7 +99,7 @@ const char* glide_status_str(glide_status s) {
 
 size_t glide_attn_workspace_bytes(const glide_attn_desc* desc, int32_t n_queries) {
   if (!desc_ok(desc) || n_queries < 1 || n_queries > glide::kMaxTree) return 0;
-  if (n_queries * (desc->H / hkv(desc)) > glide::kMaxTree) return 0;
+  if (n_queries * (desc->H / hkv(desc)) > glide::kMaxRows) return 0;
   return attn_ws_bytes(desc, n_queries);
 }
 
@@ -129,7 +129,7 @@ glide_status glide_cross_attn(const glide_attn_desc* desc, const void* q_draft, 
   // Grouped-query attention: a cached head serves H / H_kv draft queries, so
   // one pass over its keys is a small dense contraction -- the verification
   // kernels without tree keys, with the group's queries as their rows.
-  if (a.H / a.Hkv > glide::kMaxTree) return GLIDE_ERR_UNSUPPORTED;
+  if (a.H / a.Hkv > glide::kMaxRows) return GLIDE_ERR_UNSUPPORTED;
   if (!(a.flags & GLIDE_FLAG_FORCE_FMA)) {
     cudaError_t e = glide::launch_tree_attn_tc(a, st);
     if (e != cudaErrorNotSupported) return from_cuda(e);
@@ -148,7 +148,7 @@ glide_status tree_verify_attn(const glide_attn_desc* desc, const void* q_tree, i
       (reinterpret_cast<uintptr_t>(parent_idx) & 3u))
     return GLIDE_ERR_INVALID;
   if (max_kv_len < 0 || (long long)max_kv_len + n > desc->S_cap) return GLIDE_ERR_INVALID;
-  if (n * (desc->H / hkv(desc)) > glide::kMaxTree) return GLIDE_ERR_UNSUPPORTED;  // query rows of a slab
+  if (n * (desc->H / hkv(desc)) > glide::kMaxRows) return GLIDE_ERR_UNSUPPORTED;  // query rows of a slab
   if (workspace_bytes < attn_ws_bytes(desc, n)) return GLIDE_ERR_INVALID;
   glide::AttnArgs a = make_args(desc, q_tree, K_cache, V_cache, kv_len, parent_idx, out, workspace, n, max_kv_len);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

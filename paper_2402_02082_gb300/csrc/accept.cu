@@ -13,18 +13,19 @@
 //    then a warp reduction) and folds one 64-bit key (order-preserving float
 //    bits above the complemented index) into the row's slot with atomicMax.
 //    The logits are a plain HBM stream.
-// 2. every chunk is counted into its sequence's counter (release fence,
-//    atomic; nothing waits).  The warp that completes a sequence's count walks
-//    that tree: a node is accepted iff every edge on its root path matches
-//    (draft token == parent's argmax); the deepest accepted node, lowest index
-//    among equals, gives the path, its length and the bonus token.  The walk
-//    is pointer jumping over the parent array in registers (two nodes per
-//    lane, six shuffle rounds for up to 64 nodes), which gives every node its
-//    acceptance, depth and ancestor set at once.  The warp then re-arms the
-//    slots and the counter.
+// 2. every chunk is counted into its sequence's counter (release fence, then
+//    an acquire atomic; nothing waits).  The warp that completes a sequence's
+//    count walks that tree: a node is accepted iff every edge on its root
+//    path matches (draft token == parent's argmax); the deepest accepted node,
+//    lowest index among equals, gives the path, its length and the bonus
+//    token.  The walk is pointer jumping over the parent array in registers
+//    (two nodes per lane, at most six shuffle rounds for up to 64 nodes),
+//    which gives every node its acceptance, depth and ancestor set at once.
+//    The warp then re-arms the slots and the counter.
 // Because the chunk order is sequence-major and every CTA walks it in that
-// order, sequence b's chunks are all read before sequence b + 1's: the walks
-// of the early sequences run while the later ones still stream.
+// order, sequence b's chunks are all read before sequence b + 1's, and warps
+// count their chunks while they wait for the next one: the walks of the early
+// sequences run while the later ones still stream.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -34,7 +35,7 @@
 namespace glide {
 namespace {
 
-constexpr int kNW = 12;                       // consumer warps
+constexpr int kNW = 14;                       // consumer warps (14 stages of 16 KB fill the shared memory)
 constexpr int kThreads = (kNW + 1) * 32;      // + one producer warp
 constexpr int kChunk = 4096;                  // logits per chunk (16 KB)
 constexpr int kNS = kNW;                      // ring stages: stage s serves consumer warp s only
@@ -69,6 +70,14 @@ __device__ __forceinline__ int key_index(unsigned long long k) {
   return (int)(0xffffffffu - (uint32_t)(k & 0xffffffffull));
 }
 
+// Counter increment with acquire semantics: a thread that sees the final
+// count also sees every slot update fenced before the other increments.
+__device__ __forceinline__ unsigned atomic_add_acquire(unsigned* addr, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acquire.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(addr), "r"(v) : "memory");
+  return old;
+}
+
 // (value, index) pairs: the larger value wins, the lower index among equals.
 __device__ __forceinline__ void warp_argmax(float& m, int& idx) {
 #pragma unroll
@@ -97,9 +106,10 @@ __device__ __forceinline__ uint32_t pack(bool ok, int d, int p) {
   return (ok ? 0x10000u : 0u) | ((uint32_t)d << 8) | (uint32_t)(p + 1);
 }
 
-// Walks sequence b's tree (one whole warp; every chunk of b has been counted).
+// Walks sequence b's tree (one whole warp; every chunk of b has been counted,
+// and the count that completed it was an acquire by one lane of this warp).
 __device__ void walk_tree(const AccParams& p, int b, int lane) {
-  __threadfence();  // the other chunks' slot updates were fenced before their counts
+  __syncwarp();  // orders the other lanes' loads after that lane's acquire
   const int n = p.n;
   const size_t base = (size_t)b * n;
   const int c0 = lane, c1 = lane + 32;
@@ -124,10 +134,12 @@ __device__ void walk_tree(const AccParams& p, int b, int lane) {
   uint32_t m1l = 0u, m1h = h1 ? (1u << (c1 - 32)) : 0u;
 
   // Pointer jumping: each round doubles the covered part of every root path
-  // (all lanes read the previous round's values); 2^6 = 64 > any depth.
-#pragma unroll
+  // (all lanes read the previous round's values); 2^6 = 64 > any depth, and
+  // the rounds stop once every path has reached the root.
+#pragma unroll 1
   for (int r = 0; r < 6; ++r) {
     const int q0 = (int)(w0 & 0xffu) - 1, q1 = (int)(w1 & 0xffu) - 1;
+    if (!__any_sync(0xffffffffu, q0 >= 0 || q1 >= 0)) break;
     const int i0 = q0 < 0 ? 0 : q0, i1 = q1 < 0 ? 0 : q1;
     const uint32_t g0 = gather(w0, w1, i0), g1 = gather(w0, w1, i1);
     const uint32_t gl0 = gather(m0l, m1l, i0), gh0 = gather(m0h, m1h, i0);
@@ -228,7 +240,9 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
   // A warp folds each chunk's key into its row slot at once but counts its
   // chunks in later, in batches of up to 32 (one lane per chunk): one fence
   // and one round of parallel atomics per batch instead of a fence and an
-  // atomic round trip per chunk.
+  // atomic round trip per chunk.  A batch is counted when it is full, when
+  // the warp's next chunk has not landed yet (the count then costs no time)
+  // and after the warp's last chunk.
   const unsigned per_seq = (unsigned)(p.n * p.splits);
   int pend_seq = 0, npend = 0;  // lane i: the sequence of the warp's i-th uncounted chunk
   auto count_in = [&]() {
@@ -236,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
     __threadfence();  // the warp's slot updates are visible before any of its counts
     const bool mine = lane < npend;
     unsigned prev = 0;
-    if (mine) prev = atomicAdd(&p.counters[pend_seq], 1u);
+    if (mine) prev = atomic_add_acquire(&p.counters[pend_seq], 1u);
     unsigned done = __ballot_sync(0xffffffffu, mine && prev == per_seq - 1);
     while (done) {  // sequences this batch completed: walk each with the whole warp
       const int l = __ffs(done) - 1;
@@ -254,6 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
     float m = -__int_as_float(0x7f800000);  // -inf
     int idx = 0x7fffffff;                   // a lane that holds no logit never wins
     if (p.bulk) {
+      if (npend > 0 && !mbar_test_wait(&full[warp], (uint32_t)(use & 1))) count_in();
       if (!mbar_wait(&full[warp], (uint32_t)(use & 1), abort_flag, p.status)) break;
       const float4* s4 = reinterpret_cast<const float4*>(ring + (size_t)warp * kChunk);
       const int n4 = cnt >> 2;  // cnt is a multiple of 4 in this mode

@@ -193,26 +193,34 @@ __device__ __forceinline__ size_t out_row(int b, int h, int r, int nrows, int gr
   return ((size_t)b * (nrows / group) + node) * Hq + (size_t)h * group + (r - node * group);
 }
 
-// After this CTA wrote its partial for (b, h) into its slot, count the CTA in;
-// the CTA that completes the count merges every slot of (b, h) into `out` and
-// re-arms the counter.  Nothing waits: the last arrival does the work.  (b, h)
-// is a slab of cached head h; its nq query rows map to outputs by out_row.
-// Called by all `nthreads` consumer threads.
-__device__ inline void combine_if_last(const Segment& s, int B, int H, int nq, int D, int group, int Hq,
-                                       float* partials, unsigned* counters, float* out, int ctid, int nthreads,
-                                       volatile int* flag) {
+// Split-KV bookkeeping of a slab (b, cached head h) whose nq query rows are
+// served in row tiles of at most 64: each row tile has its own arrival
+// counter (index cidx, see row_tile_counter) and merges its rows [r0, r0 + nr)
+// of the partial slots.  One row tile covers all rows when nq <= 64.
+__device__ __forceinline__ int row_tile_counter(int b, int h, int H, int R, int y) {
+  return (b * H + h) * R + y;
+}
+
+// After this CTA wrote its partial rows [r0, r0 + nr) for (b, h) into its
+// slot, count the CTA in; the CTA that completes the count merges those rows
+// of every slot of (b, h) into `out` and re-arms the counter.  Nothing waits:
+// the last arrival does the work.  The slab's nq query rows map to outputs by
+// out_row.  Called by all `nthreads` consumer threads.
+__device__ inline void combine_if_last(const Segment& s, int H, int nq, int r0, int nr, int cidx, int D, int group,
+                                       int Hq, float* partials, unsigned* counters, float* out, int ctid,
+                                       int nthreads, volatile int* flag) {
   const int bh = s.b * H + s.h;
   __threadfence();
   consumer_sync(nthreads);
   if (ctid == 0) {
-    const unsigned prev = atomicAdd(&counters[bh], 1u);
+    const unsigned prev = atomicAdd(&counters[cidx], 1u);
     *flag = (prev == (unsigned)(s.c_last - s.c_first)) ? 1 : 0;
   }
   consumer_sync(nthreads);
   if (*flag) {
     __threadfence();
-    for (int idx = ctid; idx < nq * D; idx += nthreads) {
-      const int iq = idx / D, d = idx - iq * D;
+    for (int idx = ctid; idx < nr * D; idx += nthreads) {
+      const int iq = r0 + idx / D, d = idx % D;
       float M = -CUDART_INF_F;
       for (int c = s.c_first; c <= s.c_last; ++c) {
         const float* row = partial_slot(partials, c + bh, nq, D) + (size_t)iq * (D + 2);
@@ -227,21 +235,21 @@ __device__ inline void combine_if_last(const Segment& s, int B, int H, int nq, i
       }
       out[out_row(s.b, s.h, iq, nq, group, Hq) * D + d] = O / L;
     }
-    if (ctid == 0) counters[bh] = 0u;
+    if (ctid == 0) counters[cidx] = 0u;
   }
   consumer_sync(nthreads);
 }
 
-// The arrival half of combine_if_last: after this CTA wrote its partial for
-// (b, h), count it in; returns true (in every calling thread) if this CTA
-// completed the count and so must merge the (b, h) later with
-// combine_partials.  Called by all `nthreads` consumer threads.
-__device__ inline bool arrive_split(const Segment& s, int H, unsigned* counters, int ctid, int nthreads,
+// The arrival half of combine_if_last: after this CTA wrote its partial rows
+// for (b, h), count it in on counter cidx; returns true (in every calling
+// thread) if this CTA completed the count and so must merge the rows later
+// with combine_partials.  Called by all `nthreads` consumer threads.
+__device__ inline bool arrive_split(const Segment& s, int cidx, unsigned* counters, int ctid, int nthreads,
                                     volatile int* flag) {
   __threadfence();
   consumer_sync(nthreads);
   if (ctid == 0) {
-    const unsigned prev = atomicAdd(&counters[s.b * H + s.h], 1u);
+    const unsigned prev = atomicAdd(&counters[cidx], 1u);
     *flag = (prev == (unsigned)(s.c_last - s.c_first)) ? 1 : 0;
   }
   consumer_sync(nthreads);
@@ -255,28 +263,29 @@ struct OutMap {
   __device__ long long row(int b, int h, int r, int nq) const { return (long long)out_row(b, h, r, nq, group, Hq); }
 };
 
-// Merges every split partial of slab (b, h) = (s.b, s.h) into `out` (query
-// rows placed by the OutMap) and re-arms
-// the counter; all `nthreads` threads of the CTA call it (it uses
-// __syncthreads).  scratch: shared memory for (2 + kCombineW) * nq floats.
+// Merges rows [r0, r0 + nr) of every split partial of slab (b, h) =
+// (s.b, s.h) into `out` (query rows placed by the OutMap) and re-arms counter
+// cidx; all `nthreads` threads of the CTA call it (it uses __syncthreads).
+// scratch: shared memory for (2 + kCombineW) * nr floats.
 // Pass 1, one thread per query row: M = max_c m_c, the weights
 // w_c = 2^(m_c - M) and 1 / sum_c w_c l_c.  Pass 2: float4 outputs, each
 // thread taking kCombineU of them with every load issued before any use.
 constexpr int kCombineW = 8;   // slots whose weights are kept in shared memory
 constexpr int kCombineU = 3;   // outputs per thread per round
-__device__ inline void combine_partials(const Segment& s, int H, int nq, int D, const OutMap& om,
-                                        const float* partials, unsigned* counters, float* out, float* scratch,
-                                        int tid, int nthreads) {
+__device__ inline void combine_partials(const Segment& s, int H, int nq, int r0, int nr, int cidx, int D,
+                                        const OutMap& om, const float* partials, unsigned* counters, float* out,
+                                        float* scratch, int tid, int nthreads) {
   const int bh = s.b * H + s.h;
   const int nsl = s.c_last - s.c_first + 1;
   const int rs = D + 2;  // floats per partial row: m, l, o[D]
   float* Mrow = scratch;
-  float* Linv = scratch + nq;
-  float* W = scratch + 2 * nq;
-  const float* slot0 = partial_slot(const_cast<float*>(partials), s.c_first + bh, nq, D);
-  const size_t sstride = (size_t)nq * rs;  // consecutive CTAs' slots of one (b, h) are adjacent
+  float* Linv = scratch + nr;
+  float* W = scratch + 2 * nr;
+  // row r0 of the first slot; consecutive CTAs' slots of one (b, h) are adjacent
+  const float* slot0 = partial_slot(const_cast<float*>(partials), s.c_first + bh, nq, D) + (size_t)r0 * rs;
+  const size_t sstride = (size_t)nq * rs;
   __threadfence();
-  for (int r = tid; r < nq; r += nthreads) {
+  for (int r = tid; r < nr; r += nthreads) {
     // one round of loads: (m, l) of every slot, with a running max
     float M = -CUDART_INF_F, L = 0.f;
 #pragma unroll 4
@@ -300,7 +309,7 @@ __device__ inline void combine_partials(const Segment& s, int H, int nq, int D, 
   }
   __syncthreads();
   const int cpr = D / 4;
-  const int items = nq * cpr;
+  const int items = nr * cpr;
   for (int base = tid; base < items; base += kCombineU * nthreads) {
     float4 acc[kCombineU];
 #pragma unroll
@@ -356,12 +365,12 @@ __device__ inline void combine_partials(const Segment& s, int H, int nq, int D, 
       if (it < items) {
         const int r = it / cpr, d0 = (it - r * cpr) * 4;
         const float li = Linv[r];
-        *reinterpret_cast<float4*>(out + om.row(s.b, s.h, r, nq) * D + d0) =
+        *reinterpret_cast<float4*>(out + om.row(s.b, s.h, r0 + r, nq) * D + d0) =
             make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
       }
     }
   }
-  if (tid == 0) counters[bh] = 0u;
+  if (tid == 0) counters[cidx] = 0u;
   __syncthreads();
 }
 

@@ -8,6 +8,8 @@ namespace glide {
 
 constexpr int kMaxBatch = 1024;   // sequences per call (per-CTA tile table lives in shared memory)
 constexpr int kMaxTree = 64;      // tree nodes (one 64-bit ancestor mask per node)
+constexpr int kRowTile = 64;      // query rows of a slab one verification CTA serves
+constexpr int kMaxRows = 256;     // query rows per slab (n nodes x H / H_kv heads): up to four row tiles
 constexpr int kMaxCtas = 1024;    // CTAs (or claimed chunks) per attention launch (bounds the partial slots)
 constexpr int kCrossPartials = 8; // cross-attention partials per slot: one per consumer warp
 constexpr int kCapeMaxSet = 7;    // largest expansion set: S(p) <= 7, fixed sizes up to 7

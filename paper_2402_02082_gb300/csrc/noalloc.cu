@@ -16,8 +16,6 @@
 // library routine.
 #include <cuda_runtime.h>
 
-#include <mutex>
-
 #include "../../include/glide.h"
 #include "common.cuh"
 #include "kernels.h"
@@ -25,32 +23,23 @@
 namespace {
 
 constexpr size_t kScratchBytes = 32u << 20;  // 32 MiB per GPU
-constexpr int kMaxDevices = 64;
 
 // The scratch itself.  In host code this name is only a host-side stand-in
 // for the symbol, never a device address: host code obtains the real address
 // with cudaGetSymbolAddress (below) and passes that to the kernel.
 static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
-std::mutex g_mu;
-void* g_addr[kMaxDevices] = {};
-
-// Device address of g_scratch on the current device, looked up once per
-// device (the first call on each device does the lookup).
+// Device address of g_scratch in the current device's context.  Looked up on
+// every call (a lookup allocates nothing and enqueues nothing), so a context
+// that was torn down and created again, after cudaDeviceReset for instance,
+// gets the array's new address, never a stale one.  The first lookup on a
+// device loads the library's device code there.
 cudaError_t scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_mu);
-  if (g_addr[dev] == nullptr) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_scratch);
-    if (e != cudaSuccess) return e;
-    if (p == nullptr) return cudaErrorInvalidSymbol;
-    g_addr[dev] = p;
-  }
-  *out = g_addr[dev];
+  if (p == nullptr) return cudaErrorInvalidSymbol;
+  *out = p;
   return cudaSuccess;
 }
 
@@ -67,11 +56,27 @@ extern "C" glide_status glide_cross_attn_noalloc(const glide_attn_desc* desc, co
   if (need > kScratchBytes) return GLIDE_ERR_UNSUPPORTED;
   void* scratch = nullptr;
   if (scratch_address(&scratch) != cudaSuccess) return GLIDE_ERR_CUDA;
-  // The array keeps whatever the previous call left; the status word and the
-  // arrival counters must start at zero.  (cudaMemsetAsync does not allocate.)
+  // The array keeps whatever the previous call left.  The counters after the
+  // status word must start at zero; the status word itself (bytes 0..3) is
+  // left alone, so a wait that ran out in an earlier call stays reported
+  // until glide_noalloc_read_device_status reads and clears it.
+  // (cudaMemsetAsync does not allocate.)
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const size_t zeroed = glide::WsLayout::partials_off(desc->B, desc->H);
-  if (cudaMemsetAsync(scratch, 0, zeroed, st) != cudaSuccess) return GLIDE_ERR_CUDA;
+  const size_t first = glide::WsLayout::kClaimOff;
+  const size_t zeroed = glide::WsLayout::partials_off(desc->B, desc->H) - first;
+  if (cudaMemsetAsync(static_cast<unsigned char*>(scratch) + first, 0, zeroed, st) != cudaSuccess)
+    return GLIDE_ERR_CUDA;
   return glide_cross_attn(desc, q_draft, K_cache, V_cache, kv_len, max_kv_len, out, scratch, kScratchBytes,
                           stream);
+}
+
+extern "C" glide_status glide_noalloc_read_device_status(glide_stream_t stream) {
+  void* scratch = nullptr;
+  if (scratch_address(&scratch) != cudaSuccess) return GLIDE_ERR_CUDA;
+  return glide_read_device_status(scratch, stream);
+}
+
+extern "C" glide_status glide_noalloc_scratch(void** device_ptr) {
+  if (!device_ptr) return GLIDE_ERR_INVALID;
+  return scratch_address(device_ptr) == cudaSuccess ? GLIDE_OK : GLIDE_ERR_CUDA;
 }

@@ -2,8 +2,10 @@
 // (sequence, head) attend to every cached prefix key and to the tree keys of
 // their ancestors and themselves.  With grouped-query attention a slab is a
 // (sequence, cached head) and serves the n x group query rows of the heads
-// that share it (at most 64); without tree keys (prefix only) the same kernel
-// is grouped-query cross-attention.  The CaPE mask is this
+// that share it (up to kMaxRows, in row tiles of 64, one CTA per row tile:
+// the R CTAs of a share are adjacent, stream the same keys at the same time and
+// so read them from DRAM about once); without tree keys (prefix only) the same
+// kernel is grouped-query cross-attention.  The CaPE mask is this
 // ancestor-or-self mask on CaPE's trees (proposal spine plus expansion
 // leaves); the kernel takes any parent array.
 //
@@ -24,7 +26,7 @@ namespace {
 
 constexpr int kTK = 32;
 constexpr int kNW = 8;
-constexpr int kQPW = kMaxTree / kNW;  // queries per warp at most
+constexpr int kQPW = kRowTile / kNW;  // queries per warp at most
 constexpr int kThreads = (kNW + 1) * 32;
 
 template <typename T, int D>
@@ -55,7 +57,8 @@ struct TreeParams {
   int B, H, S_cap, max_kv_len, n;
   int Hkv;    // cached heads (slabs are (b, cached head))
   int group;  // query heads per cached head (H / Hkv)
-  int rows;   // query rows per slab: n nodes x group heads, node-major, <= 64
+  int rows;   // query rows per slab: n nodes x group heads, node-major, <= kMaxRows
+  int R;      // row tiles per slab: CTA x * R + y serves rows [64y, 64y + 64) of share x
   int tree;   // 1: the n tree keys follow the prefix (verification); 0: prefix only
   float scale_log2;
 };
@@ -97,9 +100,12 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
   }
 
+  // this CTA: share x of the key sequence, row tile y of every slab in it
+  const int x = blockIdx.x / p.R, y = blockIdx.x - x * p.R;
+  const int row0 = y * kRowTile, rows_here = min(kRowTile, p.rows - row0);
   Partition P;
-  P.init(bt.start[p.B], gridDim.x);
-  const long long g_begin = P.begin(blockIdx.x), g_end = P.end(blockIdx.x);
+  P.init(bt.start[p.B], gridDim.x / p.R);
+  const long long g_begin = P.begin(x), g_end = P.end(x);
   const T* Kg = static_cast<const T*>(p.K);
   const T* Vg = static_cast<const T*>(p.V);
 
@@ -155,16 +161,17 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
 
     float q[kQPW][E], o[kQPW][E], m[kQPW], l[kQPW];
     uint64_t am[kQPW];
-    // query row iq of the slab: node iq / group, head s.h * group + iq % group
+    // query row iq of the slab (row0 + warp + j * kNW): node iq / group, head
+    // s.h * group + iq % group
 #pragma unroll
     for (int j = 0; j < kQPW; ++j) {
-      const int iq = warp + j * kNW;
+      const int iq = row0 + warp + j * kNW;
       m[j] = -CUDART_INF_F;
       l[j] = 0.f;
       am[j] = 0;
 #pragma unroll
       for (int e = 0; e < E; ++e) { o[j][e] = 0.f; q[j][e] = 0.f; }
-      if (iq < p.rows) {
+      if (warp + j * kNW < rows_here) {
         const int node = iq / p.group;
         load_row_chunk<T, E>(static_cast<const T*>(p.q) + out_row(s.b, s.h, iq, p.rows, p.group, p.H) * D + lane * E,
                              q[j]);
@@ -184,7 +191,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       const T* Vt = sV + (size_t)st * kTK * D + lane * E;
 #pragma unroll
       for (int j = 0; j < kQPW; ++j) {
-        if (warp + j * kNW >= p.rows) break;
+        if (warp + j * kNW >= rows_here) break;
         float part[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
@@ -224,11 +231,11 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
 
     const int bh = s.b * p.Hkv + s.h;
     const bool single = s.c_first == s.c_last;
-    float* slot = partial_slot(p.partials, blockIdx.x + bh, p.rows, D);
+    float* slot = partial_slot(p.partials, x + bh, p.rows, D);
 #pragma unroll
     for (int j = 0; j < kQPW; ++j) {
-      const int iq = warp + j * kNW;
-      if (iq >= p.rows) break;
+      if (warp + j * kNW >= rows_here) break;
+      const int iq = row0 + warp + j * kNW;
       const float L = warp_sum(l[j]);
       if (single) {
         float* dst = p.out + out_row(s.b, s.h, iq, p.rows, p.group, p.H) * D + lane * E;
@@ -242,7 +249,8 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
       }
     }
     if (single) consumer_sync(kCT);
-    else combine_if_last(s, p.B, p.Hkv, p.rows, D, p.group, p.H, p.partials, p.counters, p.out, ctid, kCT, last_flag);
+    else combine_if_last(s, p.Hkv, p.rows, row0, rows_here, row_tile_counter(s.b, s.h, p.Hkv, p.R, y), D, p.group,
+                         p.H, p.partials, p.counters, p.out, ctid, kCT, last_flag);
     i_base += ntile;
     g = s.g_end;
   }
@@ -259,7 +267,10 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
     configured = true;
   }
   const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
-  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
+  const int rows = a.nq * (a.H / a.Hkv);
+  const int R = (rows + kRowTile - 1) / kRowTile;
+  // G shares of the key sequence, R CTAs (row tiles) per share
+  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count() / R;
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
   if (G < 1) G = 1;
@@ -270,16 +281,16 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
   p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
-  p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.rows = a.nq * p.group; p.tree = a.tree;
+  p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.rows = rows; p.R = R; p.tree = a.tree;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_fma_kernel<T, D><<<(unsigned)G, kThreads, C::smem_bytes(a.B), st>>>(p);
+  tree_attn_fma_kernel<T, D><<<(unsigned)(G * R), kThreads, C::smem_bytes(a.B), st>>>(p);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_tree_attn_fma(const AttnArgs& a, cudaStream_t st) {
-  if (a.nq * (a.H / a.Hkv) > kMaxTree) return cudaErrorInvalidValue;  // the abi rejects this first
+  if (a.nq * (a.H / a.Hkv) > kMaxRows) return cudaErrorInvalidValue;  // the abi rejects this first
   if (a.dtype == 0 && a.D == 128) return launch_typed<__nv_bfloat16, 128>(a, st);
   if (a.dtype == 0 && a.D == 64) return launch_typed<__nv_bfloat16, 64>(a, st);
   if (a.dtype == 1 && a.D == 128) return launch_typed<float, 128>(a, st);

@@ -13,6 +13,13 @@
 // (TMEM): four S buffers of 64 columns and one O accumulator of D columns for
 // each key half.
 //
+// Grouped-query slabs (a sequence's cached head and the n x H/H_kv query rows
+// it serves) with more than 64 rows are served in row tiles of 64: the grid
+// holds R CTAs per share of the key sequence, CTA x * R + y taking row tile y
+// of every slab in share x.  The R CTAs of a share are adjacent, so they run
+// together and stream the same K/V tiles at about the same time: DRAM serves
+// each tile about once and L2 the other R - 1 reads.
+//
 // Roles (384 threads, persistent grid of one CTA per SM, split-KV partition
 // shared with the other attention kernels):
 //   warps 0-7  softmax.  An M = 64 accumulator keeps rows 16q..16q+15 in
@@ -107,7 +114,8 @@ struct TcParams {
   int B, H, S_cap, max_kv_len, n;
   int Hkv;    // cached heads (slabs are (b, cached head))
   int group;  // query heads per cached head (H / Hkv)
-  int rows;   // query rows per slab: n nodes x group heads, node-major, <= 64
+  int rows;   // query rows per slab: n nodes x group heads, node-major, <= kMaxRows
+  int R;      // row tiles per slab (rows / 64 rounded up)
   int tree;   // 1: the n tree keys follow the prefix (verification); 0: prefix only
   int ns;  // K/V stages
   float scale_log2;
@@ -230,9 +238,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::fence_after_sync();
   const uint32_t tmem = *tmem_slot;
 
+  // this CTA: share x of the key sequence, row tile y of every slab in it
+  const int x = blockIdx.x / p.R, y = blockIdx.x - x * p.R;
+  const int row0 = y * kM, rows_here = min(kM, p.rows - row0);
   Partition P;
-  P.init(bt.start[p.B], gridDim.x);
-  const long long g_begin = P.begin(blockIdx.x), g_end = P.end(blockIdx.x);
+  P.init(bt.start[p.B], gridDim.x / p.R);
+  const long long g_begin = P.begin(x), g_end = P.end(x);
 
   if (warp == kProdWarp) {
     // ------------------------------------------------------------ producer
@@ -242,7 +253,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       tc::prefetch_tmap(&tmK);
       tc::prefetch_tmap(&tmV);
-      const uint64_t pol = policy_evict_first();
+      // one reader per tile: evict it first; R row tiles read each tile R times
+      const uint64_t pol = p.R == 1 ? policy_evict_first() : policy_evict_normal();
       struct Cursor {  // next tile to load: CTA-local index i, segment s, tile t
         int i, t;
         long long g;
@@ -380,9 +392,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rr = (lane >> 2) + 8 * (lane & 1);  // row within the quarter
     const int cpar = (lane >> 1) & 1;             // column parity of this thread
     const int row = quarter * 16 + rr;            // MMA row
-    const int qi = rr * 4 + quarter;              // the query row of this MMA row
-    const bool valid = qi < p.rows;
-    const int node = valid ? qi / p.group : 0;    // its tree node
+    const int qi = rr * 4 + quarter;              // the query row of this MMA row, within the row tile
+    const bool valid = qi < rows_here;
+    const int node = valid ? (row0 + qi) / p.group : 0;  // its tree node
     const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
     const uint32_t o_col = C::kTmemO + half * D;
     const int sid = threadIdx.x;                  // 0..255 among the softmax threads
@@ -398,7 +410,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto row_at = [&](const Segment& sq, int& lim) -> long long {
       lim = bt.plen[sq.b];
       if (!valid) return -1;
-      return om.row(sq.b, sq.h, qi, p.rows);
+      return om.row(sq.b, sq.h, row0 + qi, p.rows);
     };
     auto write_q = [&](const Segment& sq, int sg) {
       unsigned char* qrow = base + C::off_Q + (row >> 3) * 1024 + (row & 7) * 128;
@@ -575,7 +587,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool single = s.c_first == s.c_last;
         const int bh = s.b * p.Hkv + s.h;
         float* dst = single ? p.out + (orow >= 0 ? orow : 0) * D
-                            : partial_slot(p.partials, blockIdx.x + bh, p.rows, D) + (size_t)(valid ? qi : 0) * (D + 2) + 2;
+                            : partial_slot(p.partials, x + bh, p.rows, D) + (size_t)(row0 + (valid ? qi : 0)) * (D + 2) + 2;
         const bool write = single ? orow >= 0 : valid;
         if (!dead) {
           tc::fence_after_sync();
@@ -630,7 +642,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // after this CTA's last tile (see the end of the kernel), so that the
         // merge does not hold up the next segment.  Only the first and the last
         // segment of a CTA's share can be split.
-        if (!single && arrive_split(s, p.Hkv, p.counters, sid, kSoftWarps * 32, last_flag)) {
+        if (!single && arrive_split(s, row_tile_counter(s.b, s.h, p.Hkv, p.R, y), p.counters, sid, kSoftWarps * 32,
+                                    last_flag)) {
           if (sid == 0) pend[npend] = make_int4(s.b, s.h, s.c_first, s.c_last);
           ++npend;
         }
@@ -655,8 +668,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     Segment s;
     s.b = pend[k].x; s.h = pend[k].y; s.c_first = pend[k].z; s.c_last = pend[k].w;
     const OutMap om{p.group, p.H};
-    combine_partials(s, p.Hkv, p.rows, D, om, p.partials, p.counters, p.out, reinterpret_cast<float*>(base + C::off_P),
-                     threadIdx.x, kThreads);
+    combine_partials(s, p.Hkv, p.rows, row0, rows_here, row_tile_counter(s.b, s.h, p.Hkv, p.R, y), D, om, p.partials,
+                     p.counters, p.out, reinterpret_cast<float*>(base + C::off_P), threadIdx.x, kThreads);
   }
 }
 
@@ -682,7 +695,9 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   CUtensorMap mk, mv;
   if (!make_bf16_map(&mk, a.K, rows, D, D, kTK) || !make_bf16_map(&mv, a.V, rows, D, D, kTK)) return cudaErrorNotSupported;
   const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kTK - 1) / kTK);
-  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count();
+  const int R = (a.nq * group + kM - 1) / kM;
+  // G shares of the key sequence, R CTAs (row tiles) per share
+  long long G = a.max_ctas > 0 ? a.max_ctas : sm_count() / R;
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
   if (G < 1) G = 1;
@@ -696,10 +711,10 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
   p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
-  p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.tree = a.tree;
+  p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.R = R; p.tree = a.tree;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_tc_kernel<D><<<(unsigned)G, kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
+  tree_attn_tc_kernel<D><<<(unsigned)(G * R), kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
   return cudaGetLastError();
 }
 
@@ -708,7 +723,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st) {
   if (a.dtype != 0 || (a.D != 128 && a.D != 64)) return cudaErrorNotSupported;
   if ((long long)a.B * a.Hkv * a.S_cap > 0x7fffffffLL) return cudaErrorNotSupported;  // 32-bit TMA row coordinate
-  if (a.nq * (a.H / a.Hkv) > kM) return cudaErrorNotSupported;  // rows beyond one MMA
+  if (a.nq * (a.H / a.Hkv) > kMaxRows) return cudaErrorNotSupported;  // the abi rejects this first
   if (a.D == 128) return launch_typed<128>(a, st);
   return launch_typed<64>(a, st);
 }

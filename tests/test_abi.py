@@ -35,6 +35,10 @@ def test_exports_every_declared_symbol(L):
         assert hasattr(L, name), f"libglide.so does not export {name}"
 
 
+def test_noalloc_scratch_rejects_null(L):
+    assert L.glide_noalloc_scratch(None) == gb.GLIDE_ERR_INVALID
+
+
 def test_abi_version(L):
     assert gb.glide_abi_version() == 2
 
@@ -164,11 +168,17 @@ def test_grouped_query_descriptors(L):
         d = desc(**bad)
         assert gb.glide_attn_workspace_bytes(d, 1) == 0, bad
         assert cross(L, d) == gb.GLIDE_ERR_INVALID, bad
-    # 32 query heads over 8 cached heads: 4 rows per node; a 26-node tree needs 104 > 64 rows
+    # 32 query heads over 8 cached heads: 4 rows per node, so every tree of up to
+    # 64 nodes fits the 256 query rows a cached head can serve
     d = desc(H=32, H_kv=8)
-    assert gb.glide_attn_workspace_bytes(d, 16) > 0 and gb.glide_attn_workspace_bytes(d, 17) == 0
-    assert tree(L, d, n=17) == gb.GLIDE_ERR_UNSUPPORTED
-    assert gb.glide_attn_workspace_bytes(desc(H=128, H_kv=1), 1) == 0      # 128 heads on one cache: > 64 rows
+    assert gb.glide_attn_workspace_bytes(d, 64) > gb.glide_attn_workspace_bytes(d, 33) > 0
+    # 64 query heads over 8: 8 rows per node, 32 nodes at most
+    d = desc(H=64, H_kv=8)
+    assert gb.glide_attn_workspace_bytes(d, 32) > 0 and gb.glide_attn_workspace_bytes(d, 33) == 0
+    assert tree(L, d, n=33) == gb.GLIDE_ERR_UNSUPPORTED
+    assert gb.glide_attn_workspace_bytes(desc(H=256, H_kv=1), 1) > 0       # 256 heads on one cache: 256 rows
+    assert gb.glide_attn_workspace_bytes(desc(H=512, H_kv=1), 1) == 0      # 512 rows: beyond the limit
+    assert cross(L, desc(H=512, H_kv=1)) == gb.GLIDE_ERR_UNSUPPORTED
 
 
 def test_block_cross_attn_rejects(L):

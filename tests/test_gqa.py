@@ -47,6 +47,9 @@ def ws_for(B, H, H_kv, D, S_cap, n, dtype):
     (3, 8, 2, 64, [0, 513, 64], "bf16", 0, 0),      # an empty sequence gets zeros
     (3, 8, 2, 64, [0, 513, 64], "f32", 0, 0),       # CUDA-core path
     (1, 64, 1, 128, [2048], "bf16", 0, 0),          # one cached head for 64 query heads
+    (1, 128, 1, 128, [2048], "bf16", 0, 0),         # 128 query rows: two row tiles
+    (2, 256, 2, 64, [300, 0], "bf16", 0, 3),        # 128 rows per cached head, split shares, an empty sequence
+    (1, 256, 1, 64, [500], "f32", 0, 0),            # 256 rows on the CUDA-core path
     (4, 32, 8, 128, [4096, 100, 2000, 16], "bf16", 0, 3),     # few CTAs: split (b, h), merged
     (4, 32, 8, 128, [4096, 100, 2000, 16], "bf16", 0, 1000),
     (2, 16, 4, 128, [300, 700], "f32", 0, 7),
@@ -76,6 +79,15 @@ def test_gqa_cross_attn(B, H, H_kv, D, kv_len, dtype, flags, max_ctas):
     (1, 16, 4, 64, [777], 16, "random", "bf16", gb.GLIDE_FLAG_FORCE_FMA, 0),
     (3, 32, 8, 128, [2000, 33, 900], 6, "random", "bf16", 0, 5),
     (3, 8, 4, 64, [0, 129, 64], 9, "random", "f32", 0, 1000),
+    # CaPE-sized trees (33 nodes: 32 verified tokens plus the root) on
+    # Mistral-7B's heads: 132 query rows per cached head, three row tiles
+    (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", 0, 0),
+    (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", 0, 5),
+    (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", gb.GLIDE_FLAG_FORCE_FMA, 0),
+    (1, 32, 8, 128, [1500], 64, "random", "bf16", 0, 0),       # 256 rows: the limit
+    (1, 32, 8, 128, [1500], 64, "random", "bf16", 0, 1000),
+    (2, 16, 4, 64, [700, 65], 20, "random", "bf16", 0, 7),     # 80 rows, D = 64
+    (2, 16, 4, 64, [700, 0], 20, "random", "f32", 0, 3),
 ])
 def test_gqa_tree_verify(B, H, H_kv, D, kv_len, n, tree, dtype, flags, max_ctas):
     K, V, _, qt, parent = make(B, H, H_kv, D, kv_len, n, dtype, seed=800 + n + H, tree=tree)
