@@ -9,7 +9,10 @@ needed between steps.
 
 Prints ONE JSON line.  `value` is the KV-cache bytes the step reads
 (gamma cross-attention passes + one verification pass) divided by the device
-time of the step.  --impl reference times the fp64 CPU oracle instead.
+time of the step.  Beside it: every evaluation workload's round
+(`per_config`), whole GliDe-with-CaPE rounds with their fixed (non-attention)
+part (`cape_round`), and the calls around the round timed alone
+(`next_rows`).  --impl reference times the fp64 CPU oracle instead.
 """
 from __future__ import annotations
 
@@ -258,8 +261,446 @@ def workload_config(w):
 
 # -------------------------------------------------------------------- main
 # kernels each library call launches (cross-attention: the attention kernel and its merge)
-LAUNCHES_PER_CALL = {"glide_cross_attn": 2, "tree_verify_attn": 1, "tree_accept": 1}
+LAUNCHES_PER_CALL = {"glide_cross_attn": 2, "tree_verify_attn": 1, "tree_accept": 1, "cape_expand": 1,
+                     "glide_kv_compact": 1}
 CAPE_MAX_TOKENS = 32   # the cap on verified tokens of the paper's CaPE runs (Section 4)
+L2_BYTES = 129e6
+
+
+def event_pair():
+    import torch
+    return torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+
+class Round:
+    """One workload's speculative round resident on the device, through the
+    public API: gamma glide_cross_attn calls (the draft steps), one
+    tree_verify_attn over the workload's tree, one tree_accept.  Also the
+    pinned host copies of the per-round inputs and results for the
+    end-to-end measurement."""
+
+    def __init__(self, gb, w, dev, flags=0):
+        import torch
+        self.gb, self.w, self.dev, self.flags = gb, w, dev, flags
+        case = synth.make_case(w, garbage="zero")
+        self.case = case
+        self.K, self.V = self.to_dev(case["K"]), self.to_dev(case["V"])
+        self.q_draft = [self.to_dev(case["q_draft"][i]) for i in range(w.gamma)]
+        self.q_tree = self.to_dev(case["q_tree"])
+        self.parent = self.to_dev(case["parent_idx"].astype(np.int32))
+        self.kv_len = self.to_dev(np.asarray(w.kv_len, dtype=np.int32))
+        self.draft = self.to_dev(case["draft_tokens"].astype(np.int32))
+        self.logits = self.to_dev(case["target_logits"])
+        B, H, S_cap, D = case["K"].shape
+        self.B, self.H, self.D, self.n = B, H, D, w.n
+        desc = gb.make_desc(B, H, D, S_cap, gb.GLIDE_BF16 if w.dtype == "bf16" else gb.GLIDE_F32)
+        self.ws = torch.zeros(gb.glide_attn_workspace_bytes(desc, w.n), dtype=torch.uint8, device=dev)
+        self.ws_acc = torch.zeros(gb.glide_accept_workspace_bytes(B, w.n), dtype=torch.uint8, device=dev)
+        self.out_c = [torch.empty(B, 1, H, D, device=dev) for _ in range(w.gamma)]
+        self.out_t = torch.empty(B, w.n, H, D, device=dev)
+        self.path = torch.empty(B, w.n, dtype=torch.int32, device=dev)
+        self.ln = torch.empty(B, dtype=torch.int32, device=dev)
+        self.bonus = torch.empty(B, dtype=torch.int32, device=dev)
+        self.names = ["glide_cross_attn"] * w.gamma + ["tree_verify_attn", "tree_accept"]
+        self._host = None
+
+    def to_dev(self, a):
+        import torch
+        if a.dtype == np.uint16:
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(self.dev)
+        return torch.from_numpy(np.ascontiguousarray(a)).to(self.dev)
+
+    def calls(self, stream=None):
+        gb, w = self.gb, self.w
+        fns = [lambda i=i: gb.glide_cross_attn(self.q_draft[i], self.K, self.V, self.kv_len, w.max_kv_len,
+                                               self.out_c[i], self.ws, stream=stream) for i in range(w.gamma)]
+        fns.append(lambda: gb.tree_verify_attn(self.q_tree, self.parent, self.K, self.V, self.kv_len, w.max_kv_len,
+                                               self.out_t, self.ws, flags=self.flags, stream=stream))
+        fns.append(lambda: gb.tree_accept(self.draft, self.parent, self.logits, self.path, self.ln, self.bonus,
+                                          self.ws_acc, stream=stream))
+        return fns
+
+    def step(self):
+        for f in self.calls():
+            f()
+
+    def status_ok(self):
+        gb = self.gb
+        return gb.glide_read_device_status(self.ws) == gb.GLIDE_OK and \
+            gb.glide_read_device_status(self.ws_acc) == gb.GLIDE_OK
+
+    def kv_bytes_per_step(self):
+        cross_kv, verify_kv = kv_bytes(self.w)
+        return self.w.gamma * cross_kv + verify_kv
+
+    # ---- end to end: per-round inputs from pinned host memory, results back
+    def _pin_host(self):
+        import torch
+        w, case, n = self.w, self.case, self.w.n
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        half = lambda a: a.view(np.int16) if a.dtype == np.uint16 else a
+        h = {}
+        h["qd"] = [pin(half(case["q_draft"][i])) for i in range(w.gamma)]
+        h["qt"] = pin(half(case["q_tree"]))
+        h["par"] = pin(case["parent_idx"].astype(np.int32))
+        h["kv"] = pin(np.asarray(w.kv_len, dtype=np.int32))
+        h["dr"] = pin(case["draft_tokens"].astype(np.int32))
+        h["lg"] = pin(case["target_logits"])
+        h["tk"] = [pin(half(case["K"][b, :, w.kv_len[b]:w.kv_len[b] + n])) for b in range(self.B)]
+        h["tv"] = [pin(half(case["V"][b, :, w.kv_len[b]:w.kv_len[b] + n])) for b in range(self.B)]
+        h["rc"] = [torch.empty(self.B, 1, self.H, self.D).pin_memory() for _ in range(w.gamma)]
+        h["rt"] = torch.empty(self.B, n, self.H, self.D).pin_memory()
+        h["rp"] = torch.empty(self.B, n, dtype=torch.int32).pin_memory()
+        h["rl"] = torch.empty(self.B, dtype=torch.int32).pin_memory()
+        h["rb"] = torch.empty(self.B, dtype=torch.int32).pin_memory()
+        self._host = h
+
+    def e2e_bytes(self):
+        if self._host is None:
+            self._pin_host()
+        h = self._host
+        nb = lambda t: t.numel() * t.element_size()
+        h2d = (sum(nb(t) for t in h["qd"]) + nb(h["qt"]) + nb(h["par"]) + nb(h["kv"]) + nb(h["dr"]) + nb(h["lg"]) +
+               sum(nb(t) for t in h["tk"]) + sum(nb(t) for t in h["tv"]))
+        d2h = sum(nb(t) for t in h["rc"]) + nb(h["rt"]) + nb(h["rp"]) + nb(h["rl"]) + nb(h["rb"])
+        return h2d, d2h
+
+    def e2e_enqueue(self, s_comp, s_h2d, s_d2h):
+        """One round through the public API with host buffers, enqueued on
+        s_comp: inputs stream in on a copy stream in the order they are
+        needed, each call waits only for its own inputs, and results stream
+        back on a second copy stream, which s_comp joins at the end."""
+        import torch
+        if self._host is None:
+            self._pin_host()
+        h, w, n, gb = self._host, self.w, self.w.n, self.gb
+        bits = lambda t: t.view(torch.int16) if t.dtype == torch.bfloat16 else t
+        K16, V16 = bits(self.K), bits(self.V)
+        fork = s_comp.record_event()
+        s_h2d.wait_event(fork)
+        s_d2h.wait_event(fork)
+        ev_in = []
+        with torch.cuda.stream(s_h2d):
+            self.kv_len.copy_(h["kv"], non_blocking=True)
+            for i in range(w.gamma):
+                bits(self.q_draft[i]).copy_(h["qd"][i], non_blocking=True)
+                ev_in.append(s_h2d.record_event())
+            for b in range(self.B):
+                K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(h["tk"][b], non_blocking=True)
+                V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(h["tv"][b], non_blocking=True)
+            bits(self.q_tree).copy_(h["qt"], non_blocking=True)
+            self.parent.copy_(h["par"], non_blocking=True)
+            ev_tree = s_h2d.record_event()
+            self.draft.copy_(h["dr"], non_blocking=True)
+            self.logits.copy_(h["lg"], non_blocking=True)
+            ev_acc = s_h2d.record_event()
+
+        def back(pairs):
+            done = s_comp.record_event()
+            s_d2h.wait_event(done)
+            with torch.cuda.stream(s_d2h):
+                for dst, src in pairs:
+                    dst.copy_(src, non_blocking=True)
+
+        for i in range(w.gamma):
+            s_comp.wait_event(ev_in[i])
+            gb.glide_cross_attn(self.q_draft[i], self.K, self.V, self.kv_len, w.max_kv_len, self.out_c[i], self.ws,
+                                stream=s_comp)
+            back([(h["rc"][i], self.out_c[i])])
+        s_comp.wait_event(ev_tree)
+        gb.tree_verify_attn(self.q_tree, self.parent, self.K, self.V, self.kv_len, w.max_kv_len, self.out_t,
+                            self.ws, flags=self.flags, stream=s_comp)
+        back([(h["rt"], self.out_t)])
+        s_comp.wait_event(ev_acc)
+        gb.tree_accept(self.draft, self.parent, self.logits, self.path, self.ln, self.bonus, self.ws_acc,
+                       stream=s_comp)
+        back([(h["rp"], self.path), (h["rl"], self.ln), (h["rb"], self.bonus)])
+        s_comp.wait_event(s_d2h.record_event())
+        s_comp.wait_event(s_h2d.record_event())
+
+
+def time_e2e(enqueue, dev, steps, world):
+    """Seconds for `steps` end-to-end rounds, each enqueued by enqueue(s_comp,
+    s_h2d, s_d2h) and waited for: eager, and replayed as one CUDA graph (the
+    host then enqueues one graph instead of every copy and launch).  Returns
+    (eager_s, graph_s or None, launch description)."""
+    import torch
+    import torch.distributed as dist
+    s_comp = torch.cuda.Stream(device=dev)   # not the legacy default stream: it can be captured
+    s_h2d = torch.cuda.Stream(device=dev)
+    s_d2h = torch.cuda.Stream(device=dev)
+
+    def eager_step():
+        enqueue(s_comp, s_h2d, s_d2h)
+        s_comp.synchronize()
+
+    def timed(step):
+        for _ in range(2):
+            step()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            step()
+        return max_over_ranks(time.perf_counter() - t0, dev)
+
+    eager_s = timed(eager_step)
+    try:
+        graph = torch.cuda.CUDAGraph()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(graph, stream=s_comp):
+            enqueue(s_comp, s_h2d, s_d2h)
+        torch.cuda.synchronize()
+
+        def graph_step():
+            graph.replay()
+            torch.cuda.current_stream().synchronize()
+        return eager_s, timed(graph_step), "cuda_graph"
+    except Exception as exc:  # capture refused on this stack: the eager round is the number
+        return eager_s, None, f"eager (graph capture failed: {type(exc).__name__})"
+
+
+def time_steps_events(step, steps, flush=None):
+    """CUDA-event time (ms) of each of `steps` calls of step() on the current
+    stream; with `flush`, a buffer larger than L2 is written before every step
+    (outside the timed span)."""
+    import torch
+    stream = torch.cuda.current_stream()
+    spans = []
+    for _ in range(steps):
+        if flush is not None:
+            flush.zero_()
+        a, b = event_pair()
+        a.record(stream)
+        step()
+        b.record(stream)
+        spans.append((a, b))
+    torch.cuda.synchronize()
+    return [a.elapsed_time(b) for a, b in spans]
+
+
+def per_config_rows(args, gb, dev, peak, head_name, head_row):
+    """Every evaluation workload's round (gamma cross-attention calls, the
+    verification and the acceptance), device-timed with CUDA events, and end
+    to end through the public API with host buffers.  Workloads whose K/V
+    fit in twice the L2 get L2 flushed (a 512 MB write) before every round."""
+    import torch
+    rows = {}
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+    for w in synth.workloads():
+        if w.name == head_name:
+            rows[w.name] = head_row
+            continue
+        r = Round(gb, w, dev)
+        for _ in range(3):
+            r.step()
+        torch.cuda.synchronize()
+        if not r.status_ok():
+            raise RuntimeError(f"device status not OK on {w.name}")
+        small = sum(kv_bytes(w)) <= 2 * L2_BYTES
+        fl = flush if small else None
+        ms = time_steps_events(r.step, args.config_steps, fl)
+        calls = {}
+        for nm, f in zip(r.names, r.calls()):
+            calls.setdefault(nm, []).extend(time_steps_events(f, max(3, args.config_steps // 3), fl))
+        step_kv = r.kv_bytes_per_step()
+        round_s = statistics.mean(ms) * 1e-3
+        eager_s, graph_s, launch = time_e2e(r.e2e_enqueue, dev, args.config_steps, 1)
+        e2e_s = (graph_s if graph_s is not None else eager_s) / args.config_steps
+        h2d, d2h = r.e2e_bytes()
+        rows[w.name] = {
+            "round_us": 1e6 * round_s, "kv_bytes_per_round": step_kv, "kv_gbs": step_kv / round_s / 1e9,
+            "frac_of_measured_hbm": step_kv / round_s / 1e9 / peak,
+            "tree_tokens_per_s_per_layer": w.B * w.n / round_s,
+            "calls_us": {k: 1e3 * statistics.mean(v) for k, v in calls.items()},
+            "e2e": {"round_us": 1e6 * e2e_s, "kv_gbs": step_kv / e2e_s / 1e9, "h2d_bytes_per_round": h2d,
+                    "d2h_bytes_per_round": d2h, "launch": launch},
+            "l2": "flushed before every round" if small else "K/V larger than twice L2 (no flush)",
+            "shape": workload_config(w)}
+        if not r.status_ok():
+            raise RuntimeError(f"device status not OK on {w.name}")
+        del r
+        torch.cuda.empty_cache()
+    del flush
+    return rows
+
+
+def time_cape_round(args, gb, dev, peak, name):
+    """A whole GliDe-with-CaPE round on one target layer of workload `name`,
+    with the tree CaPE builds: gamma glide_cross_attn calls (the draft steps),
+    cape_expand over the draft's distributions (cap of 32 verified tokens, so
+    33 tree nodes), tree_verify_attn over that tree, tree_accept, and
+    glide_kv_compact of the accepted path.  Target logits plant the first
+    four proposal tokens as argmax, so four tokens are accepted per sequence
+    (the 3-4 tokens per round of the paper's CaPE runs) and compaction moves
+    rows.  Device-timed (CUDA events around the round, and around the chain
+    expand -> verify -> accept -> compact), L2 flushed before every round when
+    the K/V fit in twice the L2; the round's fixed part is the chain less the
+    verification alone.  End to end: the round's inputs from pinned host
+    memory, its results back, replayed as one CUDA graph."""
+    import torch
+    w0 = synth.workload(name)
+    n = 1 + CAPE_MAX_TOKENS
+    w = dataclasses.replace(w0, name=f"{w0.name}-cape", n=n, gamma=max(w0.gamma, 5))
+    B, H, D = w.B, w.H, w.D
+    case = synth.make_case(w, garbage="zero")
+    to = lambda a: (torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+                    if a.dtype == np.uint16 else torch.from_numpy(np.ascontiguousarray(a)).to(dev))
+    K, V = to(case["K"]), to(case["V"])
+    S_cap = case["K"].shape[2]
+    q_draft = [to(case["q_draft"][i]) for i in range(w.gamma)]
+    q_tree = to(case["q_tree"])
+    kv_len = to(np.asarray(w.kv_len, dtype=np.int32))
+    probs_h = synth.draft_probs(w.seed + 21, B, w.gamma, w.vocab)
+    roots_h = synth.root_tokens(w.seed + 21, B, w.vocab)
+    probs, roots = to(probs_h), to(roots_h)
+    desc = gb.make_desc(B, H, D, S_cap, gb.GLIDE_BF16)
+    ws = torch.zeros(gb.glide_attn_workspace_bytes(desc, n), dtype=torch.uint8, device=dev)
+    ws_acc = torch.zeros(gb.glide_accept_workspace_bytes(B, n), dtype=torch.uint8, device=dev)
+    ws_c = torch.zeros(gb.glide_cape_workspace_bytes(B, w.gamma, w.vocab), dtype=torch.uint8, device=dev)
+    out_c = [torch.empty(B, 1, H, D, device=dev) for _ in range(w.gamma)]
+    out_t = torch.empty(B, n, H, D, device=dev)
+    tok = torch.empty(B, n, dtype=torch.int32, device=dev)
+    par = torch.empty(B, n, dtype=torch.int32, device=dev)
+    nn = torch.empty(B, dtype=torch.int32, device=dev)
+    path = torch.empty(B, n, dtype=torch.int32, device=dev)
+    ln = torch.empty(B, dtype=torch.int32, device=dev)
+    bonus = torch.empty(B, dtype=torch.int32, device=dev)
+    new_len = torch.empty(B, dtype=torch.int32, device=dev)
+    # the tree CaPE builds (the same every round), and logits that accept its
+    # first four proposal tokens
+    gb.cape_expand(probs, roots, CAPE_MAX_TOKENS, tok, par, nn, ws_c)
+    torch.cuda.synchronize()
+    tok_h = tok.cpu().numpy()
+    g = np.random.default_rng(w.seed + 22)
+    lg_h = g.standard_normal((B, n, w.vocab), dtype=np.float32)
+    for b in range(B):
+        for i in range(1, 5):   # nodes 1..gamma are the proposal x_{t+1..t+gamma}, node i's parent is i - 1
+            lg_h[b, i - 1, tok_h[b, i]] = lg_h[b, i - 1].max() + 1.0
+    logits = to(lg_h)
+
+    def expand():
+        gb.cape_expand(probs, roots, CAPE_MAX_TOKENS, tok, par, nn, ws_c)
+
+    def verify():
+        gb.tree_verify_attn(q_tree, par, K, V, kv_len, w.max_kv_len, out_t, ws)
+
+    def accept():
+        gb.tree_accept(tok, par, logits, path, ln, bonus, ws_acc)
+
+    def compact():
+        gb.glide_kv_compact(K, V, kv_len, path, ln, new_len)
+
+    def draft_steps():
+        for i in range(w.gamma):
+            gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws)
+
+    def chain():
+        expand()
+        verify()
+        accept()
+        compact()
+
+    def whole():
+        draft_steps()
+        chain()
+
+    for _ in range(3):
+        whole()
+    torch.cuda.synchronize()
+    accepted = [int(x) for x in ln.cpu().tolist()]
+    small = sum(kv_bytes(w)) <= 2 * L2_BYTES
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if small else None
+    steps = args.config_steps
+    t_round = statistics.mean(time_steps_events(whole, steps, flush))
+    t_chain = statistics.mean(time_steps_events(chain, steps, flush))
+    t_verify = statistics.mean(time_steps_events(verify, steps, flush))
+    t_draft = statistics.mean(time_steps_events(draft_steps, steps, flush))
+    for wsx in (ws, ws_acc, ws_c):
+        if gb.glide_read_device_status(wsx) != gb.GLIDE_OK:
+            raise RuntimeError("device status not OK in the CaPE round")
+
+    # end to end: the draft queries, draft distributions, roots, tree queries,
+    # the tree's own K/V rows, kv_len and the target logits come from pinned
+    # host memory; the attention outputs, the accepted path and the new
+    # lengths go back
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    half = lambda a: a.view(np.int16) if a.dtype == np.uint16 else a
+    h_qd = [pin(half(case["q_draft"][i])) for i in range(w.gamma)]
+    h_qt, h_pr, h_rt = pin(half(case["q_tree"])), pin(probs_h), pin(roots_h)
+    h_kv, h_lg = pin(np.asarray(w.kv_len, dtype=np.int32)), pin(lg_h)
+    h_tk = [pin(half(case["K"][b, :, w.kv_len[b]:w.kv_len[b] + n])) for b in range(B)]
+    h_tv = [pin(half(case["V"][b, :, w.kv_len[b]:w.kv_len[b] + n])) for b in range(B)]
+    r_c = [torch.empty(B, 1, H, D).pin_memory() for _ in range(w.gamma)]
+    r_t = torch.empty(B, n, H, D).pin_memory()
+    r_p = torch.empty(B, n, dtype=torch.int32).pin_memory()
+    r_l, r_b, r_n = (torch.empty(B, dtype=torch.int32).pin_memory() for _ in range(3))
+    bits = lambda t: t.view(torch.int16) if t.dtype == torch.bfloat16 else t
+    K16, V16 = bits(K), bits(V)
+
+    def enqueue(s_comp, s_h2d, s_d2h):
+        fork = s_comp.record_event()
+        s_h2d.wait_event(fork)
+        s_d2h.wait_event(fork)
+        ev = []
+        with torch.cuda.stream(s_h2d):
+            kv_len.copy_(h_kv, non_blocking=True)
+            for i in range(w.gamma):
+                bits(q_draft[i]).copy_(h_qd[i], non_blocking=True)
+                ev.append(s_h2d.record_event())
+            probs.copy_(h_pr, non_blocking=True)
+            roots.copy_(h_rt, non_blocking=True)
+            ev_exp = s_h2d.record_event()
+            for b in range(B):
+                K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(h_tk[b], non_blocking=True)
+                V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(h_tv[b], non_blocking=True)
+            bits(q_tree).copy_(h_qt, non_blocking=True)
+            ev_tree = s_h2d.record_event()
+            logits.copy_(h_lg, non_blocking=True)
+            ev_acc = s_h2d.record_event()
+
+        def back(pairs):
+            done = s_comp.record_event()
+            s_d2h.wait_event(done)
+            with torch.cuda.stream(s_d2h):
+                for dst, src in pairs:
+                    dst.copy_(src, non_blocking=True)
+
+        with torch.cuda.stream(s_comp):
+            for i in range(w.gamma):
+                s_comp.wait_event(ev[i])
+                gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws, stream=s_comp)
+                back([(r_c[i], out_c[i])])
+            s_comp.wait_event(ev_exp)
+            gb.cape_expand(probs, roots, CAPE_MAX_TOKENS, tok, par, nn, ws_c, stream=s_comp)
+            s_comp.wait_event(ev_tree)
+            gb.tree_verify_attn(q_tree, par, K, V, kv_len, w.max_kv_len, out_t, ws, stream=s_comp)
+            back([(r_t, out_t)])
+            s_comp.wait_event(ev_acc)
+            gb.tree_accept(tok, par, logits, path, ln, bonus, ws_acc, stream=s_comp)
+            gb.glide_kv_compact(K, V, kv_len, path, ln, new_len, stream=s_comp)
+            back([(r_p, path), (r_l, ln), (r_b, bonus), (r_n, new_len)])
+        s_comp.wait_event(s_d2h.record_event())
+        s_comp.wait_event(s_h2d.record_event())
+
+    eager_s, graph_s, launch = time_e2e(enqueue, dev, steps, 1)
+    e2e_us = 1e6 * (graph_s if graph_s is not None else eager_s) / steps
+    nb = lambda t: t.numel() * t.element_size()
+    h2d = (sum(nb(t) for t in h_qd) + nb(h_qt) + nb(h_pr) + nb(h_rt) + nb(h_kv) + nb(h_lg) +
+           sum(nb(t) for t in h_tk) + sum(nb(t) for t in h_tv))
+    d2h = sum(nb(t) for t in r_c) + nb(r_t) + nb(r_p) + 3 * nb(r_l)
+    step_kv = sum(kv_bytes(w)[0] for _ in range(w.gamma)) + kv_bytes(w)[1]
+    del K, V, flush
+    torch.cuda.empty_cache()
+    return {"round_us": 1e3 * t_round, "draft_steps_us": 1e3 * t_draft, "chain_us": 1e3 * t_chain,
+            "verify_us": 1e3 * t_verify, "fixed_us": 1e3 * (t_chain - t_verify),
+            "kv_gbs": step_kv / (t_round * 1e-3) / 1e9, "frac_of_measured_hbm": step_kv / (t_round * 1e-3) / 1e9 / peak,
+            "accepted": accepted, "tree_nodes": n,
+            "e2e": {"round_us": e2e_us, "kv_gbs": step_kv / (e2e_us * 1e-6) / 1e9, "h2d_bytes_per_round": h2d,
+                    "d2h_bytes_per_round": d2h, "launch": launch},
+            "l2": "flushed before every round" if small else "K/V larger than twice L2 (no flush)",
+            "shape": f"B={B} H={H} D={D} kv_len={list(w.kv_len)} gamma={w.gamma} V={w.vocab}, "
+                     f"CaPE tree of {n} nodes (cap {CAPE_MAX_TOKENS}), one layer"}
 
 
 def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
@@ -272,16 +713,7 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)   # > 129 MB L2
 
     def timed(fn):
-        times = []
-        for _ in range(iters + 2):
-            flush.zero_()
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            fn()
-            b.record(stream)
-            times.append((a, b))
-        torch.cuda.synchronize()
-        ms = [a.elapsed_time(b) for a, b in times[2:]]
+        ms = time_steps_events(fn, iters + 2, flush)[2:]
         return sum(ms) / len(ms)
 
     B = w.B
@@ -425,54 +857,21 @@ def run_glide(args, rank, world, local_rank):
         pool = make_pool(cores)   # spawned before any GPU work
         cpu = (pool, cores)
 
-    case = synth.make_case(w, garbage="zero")
-
-    def to_dev(a):
-        if a.dtype == np.uint16:
-            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
-        return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
-
-    K, V = to_dev(case["K"]), to_dev(case["V"])
-    q_draft = [to_dev(case["q_draft"][i]) for i in range(w.gamma)]
-    q_tree = to_dev(case["q_tree"])
-    parent = to_dev(case["parent_idx"].astype(np.int32))
-    kv_len = to_dev(np.asarray(w.kv_len, dtype=np.int32))
-    draft = to_dev(case["draft_tokens"].astype(np.int32))
-    logits = to_dev(case["target_logits"])
-    B, H, S_cap, D = case["K"].shape
-    n = w.n
-    desc = gb.make_desc(B, H, D, S_cap, gb.GLIDE_BF16 if w.dtype == "bf16" else gb.GLIDE_F32)
-    ws = torch.zeros(gb.glide_attn_workspace_bytes(desc, n), dtype=torch.uint8, device=dev)
-    ws_acc = torch.zeros(gb.glide_accept_workspace_bytes(B, n), dtype=torch.uint8, device=dev)
-    out_c = [torch.empty(B, 1, H, D, device=dev) for _ in range(w.gamma)]
-    out_t = torch.empty(B, n, H, D, device=dev)
-    path = torch.empty(B, n, dtype=torch.int32, device=dev)
-    ln = torch.empty(B, dtype=torch.int32, device=dev)
-    bonus = torch.empty(B, dtype=torch.int32, device=dev)
-    flags = gb.GLIDE_FLAG_FORCE_FMA if args.force_fma else 0
-
-    names = ["glide_cross_attn"] * w.gamma + ["tree_verify_attn", "tree_accept"]
-
-    def launches():
-        for i in range(w.gamma):
-            yield lambda i=i: gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws)
-        yield lambda: gb.tree_verify_attn(q_tree, parent, K, V, kv_len, w.max_kv_len, out_t, ws, flags=flags)
-        yield lambda: gb.tree_accept(draft, parent, logits, path, ln, bonus, ws_acc)
-
-    step_fns = list(launches())
+    r = Round(gb, w, dev, gb.GLIDE_FLAG_FORCE_FMA if args.force_fma else 0)
+    B, H, n = r.B, r.H, r.n
+    step_fns = r.calls()
+    names = r.names
     stream = torch.cuda.current_stream()
 
     for _ in range(args.warmup):
-        for f in step_fns:
-            f()
+        r.step()
     torch.cuda.synchronize()
-    if gb.glide_read_device_status(ws) != gb.GLIDE_OK or gb.glide_read_device_status(ws_acc) != gb.GLIDE_OK:
+    if not r.status_ok():
         raise RuntimeError("device status not OK after warm-up")
 
     # ---- device-timed region: inputs resident in HBM
-    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in step_fns]
-          for _ in range(args.steps)]
-    t_begin, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev = [[event_pair() for _ in step_fns] for _ in range(args.steps)]
+    t_begin, t_end = event_pair()
     clocks = ClockSampler(local_rank)
     if world > 1:
         dist.barrier()
@@ -495,131 +894,27 @@ def run_glide(args, rank, world, local_rank):
     for j, nm in enumerate(names):
         per_kernel.setdefault(nm, []).extend(ev[s][j][0].elapsed_time(ev[s][j][1]) for s in range(args.steps))
     elapsed_ms = max_over_ranks(elapsed_ms, dev)
-    if gb.glide_read_device_status(ws) != gb.GLIDE_OK or gb.glide_read_device_status(ws_acc) != gb.GLIDE_OK:
+    if not r.status_ok():
         raise RuntimeError("device status not OK after the timed region")
 
-    cross_kv, verify_kv = kv_bytes(w)
-    step_kv = w.gamma * cross_kv + verify_kv
+    step_kv = r.kv_bytes_per_step()
     value = job_throughput(step_kv * args.steps, world, elapsed_ms * 1e-3) / 1e9
     tree_tok = job_throughput(B * n * args.steps, world, elapsed_ms * 1e-3)
 
     # ---- end to end: per-round inputs from pinned host memory, results back to host
     e2e_steps = max(3, min(args.steps, args.e2e_steps))
-    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
-    h_qd = [pin(case["q_draft"][i].view(np.int16)) for i in range(w.gamma)]
-    h_qt = pin(case["q_tree"].view(np.int16) if case["q_tree"].dtype == np.uint16 else case["q_tree"])
-    h_par = pin(case["parent_idx"].astype(np.int32))
-    h_kv = pin(np.asarray(w.kv_len, dtype=np.int32))
-    h_dr = pin(case["draft_tokens"].astype(np.int32))
-    h_lg = pin(case["target_logits"])
-    tk = [pin(case["K"][b, :, w.kv_len[b]:w.kv_len[b] + n].view(np.int16)) for b in range(B)]
-    tv = [pin(case["V"][b, :, w.kv_len[b]:w.kv_len[b] + n].view(np.int16)) for b in range(B)]
-    r_c = [torch.empty(B, 1, H, D).pin_memory() for _ in range(w.gamma)]
-    r_t = torch.empty(B, n, H, D).pin_memory()
-    r_p = torch.empty(B, n, dtype=torch.int32).pin_memory()
-    r_l = torch.empty(B, dtype=torch.int32).pin_memory()
-    r_b = torch.empty(B, dtype=torch.int32).pin_memory()
-    K16, V16 = K.view(torch.int16), V.view(torch.int16)
-
-    s_comp = torch.cuda.Stream(device=dev)   # not the legacy default stream: it can be captured
-    s_h2d = torch.cuda.Stream(device=dev)
-    s_d2h = torch.cuda.Stream(device=dev)
-
-    def e2e_enqueue():
-        """One round through the public API with host buffers, enqueued on
-        s_comp: inputs stream in on a copy stream in the order they are
-        needed, each call waits only for its own inputs, and results stream
-        back on a second copy stream, which s_comp joins at the end."""
-        fork = s_comp.record_event()
-        s_h2d.wait_event(fork)
-        s_d2h.wait_event(fork)
-        ev_in = []
-        with torch.cuda.stream(s_h2d):
-            kv_len.copy_(h_kv, non_blocking=True)
-            for i in range(w.gamma):
-                q_draft[i].view(torch.int16).copy_(h_qd[i], non_blocking=True)
-                ev_in.append(s_h2d.record_event())
-            for b in range(B):
-                K16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tk[b], non_blocking=True)
-                V16[b, :, w.kv_len[b]:w.kv_len[b] + n].copy_(tv[b], non_blocking=True)
-            q_tree.view(torch.int16).copy_(h_qt, non_blocking=True)
-            parent.copy_(h_par, non_blocking=True)
-            ev_tree = s_h2d.record_event()
-            draft.copy_(h_dr, non_blocking=True)
-            logits.copy_(h_lg, non_blocking=True)
-            ev_acc = s_h2d.record_event()
-        for i in range(w.gamma):
-            s_comp.wait_event(ev_in[i])
-            gb.glide_cross_attn(q_draft[i], K, V, kv_len, w.max_kv_len, out_c[i], ws, stream=s_comp)
-            done = s_comp.record_event()
-            s_d2h.wait_event(done)
-            with torch.cuda.stream(s_d2h):
-                r_c[i].copy_(out_c[i], non_blocking=True)
-        s_comp.wait_event(ev_tree)
-        gb.tree_verify_attn(q_tree, parent, K, V, kv_len, w.max_kv_len, out_t, ws, flags=flags, stream=s_comp)
-        done = s_comp.record_event()
-        s_d2h.wait_event(done)
-        with torch.cuda.stream(s_d2h):
-            r_t.copy_(out_t, non_blocking=True)
-        s_comp.wait_event(ev_acc)
-        gb.tree_accept(draft, parent, logits, path, ln, bonus, ws_acc, stream=s_comp)
-        done = s_comp.record_event()
-        s_d2h.wait_event(done)
-        with torch.cuda.stream(s_d2h):
-            r_p.copy_(path, non_blocking=True)
-            r_l.copy_(ln, non_blocking=True)
-            r_b.copy_(bonus, non_blocking=True)
-        s_comp.wait_event(s_d2h.record_event())
-        s_comp.wait_event(s_h2d.record_event())
-
-    def eager_step():
-        e2e_enqueue()
-        s_comp.synchronize()
-
-    h2d = (sum(t.numel() * t.element_size() for t in h_qd) + h_qt.numel() * h_qt.element_size() +
-           h_par.numel() * 4 + h_kv.numel() * 4 + h_dr.numel() * 4 + h_lg.numel() * 4 +
-           sum(t.numel() * 2 for t in tk) + sum(t.numel() * 2 for t in tv))
-    d2h = sum(t.numel() * 4 for t in r_c) + r_t.numel() * 4 + r_p.numel() * 4 + 8 * B
-
-    def time_steps(step):
-        for _ in range(2):
-            step()
-        if world > 1:
-            dist.barrier()
-        t0 = time.perf_counter()
-        for _ in range(e2e_steps):
-            step()
-        return max_over_ranks(time.perf_counter() - t0, dev)
-
-    e2e_eager_s = time_steps(eager_step)
-    # The same round captured once as a CUDA graph: every step replays it (all
-    # of its copies and launches) and waits for it, so the host enqueues one
-    # graph instead of ~25 copies and launches between dependent rounds.
-    e2e_launch = "cuda_graph"
-    try:
-        graph = torch.cuda.CUDAGraph()
-        torch.cuda.synchronize()
-        with torch.cuda.graph(graph, stream=s_comp):
-            e2e_enqueue()
-        torch.cuda.synchronize()
-
-        def graph_step():
-            graph.replay()
-            torch.cuda.current_stream().synchronize()
-        e2e_s = time_steps(graph_step)
-    except Exception as exc:  # capture refused on this stack: the eager round is the number
-        e2e_launch = f"eager (graph capture failed: {type(exc).__name__})"
-        e2e_s = e2e_eager_s
+    e2e_eager_s, e2e_graph_s, e2e_launch = time_e2e(r.e2e_enqueue, dev, e2e_steps, world)
+    e2e_s = e2e_graph_s if e2e_graph_s is not None else e2e_eager_s
     e2e_value = job_throughput(step_kv * e2e_steps, world, e2e_s) / 1e9
     e2e_eager = job_throughput(step_kv * e2e_steps, world, e2e_eager_s) / 1e9
+    h2d, d2h = r.e2e_bytes()
 
-    # ---- the calls around the round: CaPE expansion (before verification) and
-    # the cache update (after acceptance), each timed alone with L2 flushed
+    # ---- the calls around the round (each timed alone with L2 flushed), every
+    # evaluation workload's round, and whole CaPE rounds
     peak, peak_src = measured_peaks()
-    next_rows = time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak)
+    next_rows = time_next_rows(args, w, r.case, gb, dev, stream, r.K, r.V, r.kv_len, peak)
 
     # ---- roofline of the dominant kernel
-
     ab = algo_bytes(w)
     kernels = {}
     for nm, times in per_kernel.items():
@@ -633,11 +928,26 @@ def run_glide(args, rank, world, local_rank):
             "peak_source": peak_src, "unit": "GB/s", "frac": kernels[dom]["frac_of_peak"],
             "traffic": recorded_traffic(dom, w.name)}
 
+    per_config, cape_round = None, None
+    if world == 1 and not args.no_per_config:
+        round_s = elapsed_ms * 1e-3 / args.steps
+        head = {"round_us": 1e6 * round_s, "kv_bytes_per_round": step_kv, "kv_gbs": step_kv / round_s / 1e9,
+                "frac_of_measured_hbm": step_kv / round_s / 1e9 / peak,
+                "tree_tokens_per_s_per_layer": B * n / round_s,
+                "calls_us": {k: v["avg_us"] for k, v in kernels.items()},
+                "e2e": {"round_us": 1e6 * e2e_s / e2e_steps, "kv_gbs": step_kv / (e2e_s / e2e_steps) / 1e9,
+                        "h2d_bytes_per_round": h2d, "d2h_bytes_per_round": d2h, "launch": e2e_launch},
+                "l2": "K/V larger than twice L2 (no flush)", "shape": workload_config(w),
+                "note": "the headline measurement above"}
+        per_config = per_config_rows(args, gb, dev, peak, w.name, head)
+        cape_round = {nm: time_cape_round(args, gb, dev, peak, nm)
+                      for nm in dict.fromkeys(("vicuna7b-chain", args.workload))}
+
     cpu_baseline = None
     if cpu is not None:
         pool, cores = cpu
         pairs = pick_pairs(w, args.cpu_pairs or w.B * w.H, 1234)
-        gbs, dt = time_oracle(w, case, pairs, pool, cores)
+        gbs, dt = time_oracle(w, r.case, pairs, pool, cores)
         pool.close()
         cpu_baseline = {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle",
                         "sample": f"{len(pairs)} of {B * H} (b,h) slabs: gamma={w.gamma} cross-attention calls + "
@@ -652,7 +962,8 @@ def run_glide(args, rank, world, local_rank):
                 "frac_of_nominal_8tbs": value / world / NOMINAL_HBM_GBS,
                 "frac_of_measured_hbm": value / world / peak,
                 "tree_tokens_per_s_per_layer": tree_tok,
-                "roofline": roof, "kernels": kernels, "next_rows": next_rows, "cpu_baseline": cpu_baseline,
+                "roofline": roof, "kernels": kernels, "per_config": per_config, "cape_round": cape_round,
+                "next_rows": next_rows, "cpu_baseline": cpu_baseline,
                 "e2e": {"value": e2e_value, "unit": "GB/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                         "steps": e2e_steps, "launch": e2e_launch, "eager_value": e2e_eager},
                 "gpu_launches": sum(LAUNCHES_PER_CALL[nm] for nm in names) * args.steps, "clocks": clk}
@@ -677,6 +988,10 @@ def main():
     ap.add_argument("--cpu-pairs", type=int, default=0,
                     help="(b, h) slabs in the CPU-baseline sample; 0 = every slab of one step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--config-steps", type=int, default=30,
+                    help="timed rounds of each evaluation workload and of the CaPE rounds")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the per-workload rounds and the CaPE rounds")
     ap.add_argument("--force-fma", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="keep only the first N sequences of the workload (smaller profiling captures)")

@@ -2,6 +2,9 @@
 through the binding, and compare with the oracle under the stated tolerance."""
 from __future__ import annotations
 
+import multiprocessing as mp
+import os
+
 import numpy as np
 import torch
 
@@ -106,3 +109,39 @@ def sample_pairs(B, H, k, seed=0):
     while len(pairs) < min(k, B * H):
         pairs.add((int(g.integers(B)), int(g.integers(H))))
     return sorted(pairs)
+
+
+def _oracle_slab(args):
+    """Oracle outputs of one (sequence, head) slab: the gamma cross-attention
+    steps and the tree verification over that slab's keys and values."""
+    import oracle
+    q_draft, q_tree, parent, Kbh, Vbh, L = args
+    cross = np.stack([oracle.cross_attn(q_draft[i][None, None, None, :], Kbh[None, None], Vbh[None, None], [L])[0, 0, 0]
+                      for i in range(q_draft.shape[0])])
+    tree = oracle.tree_verify_attn(q_tree[None, :, None, :], parent[None], Kbh[None, None], Vbh[None, None], [L])[0, :, 0]
+    return cross, tree
+
+
+def oracle_every_slab(case: dict, workers: int = 0):
+    """The oracle over every (b, h) slab of a case, spread over spawned
+    single-threaded worker processes (spawned, so the CUDA context of this
+    process is never forked).  Returns (cross [gamma, B, 1, H, D],
+    tree [B, n, H, D]) in fp64."""
+    K = case["K"]
+    B, H, _, D = K.shape
+    n = case["q_tree"].shape[1]
+    gamma = case["q_draft"].shape[0]
+    kv = [int(x) for x in case["kv_len"]]
+    args = [(case["q_draft"][:, b, 0, h, :], case["q_tree"][b, :, h, :], case["parent_idx"][b],
+             np.ascontiguousarray(K[b, h, :kv[b] + n]), np.ascontiguousarray(case["V"][b, h, :kv[b] + n]), kv[b])
+            for b in range(B) for h in range(H)]
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
+    with mp.get_context("spawn").Pool(workers or os.cpu_count() or 1) as pool:
+        res = pool.map(_oracle_slab, args, chunksize=1)
+    cross = np.zeros((gamma, B, 1, H, D))
+    tree = np.zeros((B, n, H, D))
+    for (b, h), (c, t) in zip([(b, h) for b in range(B) for h in range(H)], res):
+        cross[:, b, 0, h, :] = c
+        tree[b, :, h, :] = t
+    return cross, tree
