@@ -201,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
   __syncthreads();
   // Launched as a programmatic dependent: the inputs may come from the kernel
   // before this one, so nothing is read until that kernel has completed.
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  pdl_wait();
 
   const long long G = gridDim.x, c = blockIdx.x;
   if (warp == kNW) {
@@ -373,17 +373,7 @@ cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st) {
   if ((long long)a.n * p.splits > 0x7fffffffLL) return cudaErrorInvalidValue;
   long long G = sm_count();
   if (G > p.nchunks) G = p.nchunks;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)G);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, tree_accept_kernel, p);
+  return launch_pdl(tree_accept_kernel, dim3((unsigned)G), dim3(kThreads), kSmemBytes, st, p);
 }
 
 }  // namespace glide

@@ -130,6 +130,7 @@ __global__ void __launch_bounds__(kThreads) cape_expand_kernel(const CapeParams 
   __shared__ int s_coff[kMaxPos];              // first candidate of each position
   __shared__ int s_off[kMaxPos];               // first node of each kept set, minus 1 + gamma
   __shared__ int s_ncand, s_nodes;
+  pdl_wait();
 
   const int row = blockIdx.x / p.splits;
   const int split = blockIdx.x - row * p.splits;
@@ -338,8 +339,7 @@ cudaError_t launch_cape_expand(const CapeArgs& a, cudaStream_t st) {
   p.slots = reinterpret_cast<u64*>(ws + off);
   const long long grid = (long long)rows * p.splits;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
-  cape_expand_kernel<<<(unsigned)grid, kThreads, 0, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(cape_expand_kernel, dim3((unsigned)grid), dim3(kThreads), 0, st, p);
 }
 
 }  // namespace glide

@@ -87,6 +87,7 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
   using C = CrossCfg<T, D>;
   using G = GroupMap<T, D>;
   constexpr int NS = C::NS;
+  pdl_wait();
   extern __shared__ __align__(1024) unsigned char smem[];
   T* sK = reinterpret_cast<T*>(smem + C::off_K);
   T* sV = reinterpret_cast<T*>(smem + C::off_V);
@@ -349,7 +350,7 @@ __global__ void __launch_bounds__(kMergeWarps * 32) cross_merge_kernel(const int
   constexpr int kCols = D / 32;
   __shared__ float red[kMergeWarps][D];
   __shared__ float stat[2][kMergeWarps];
-  asm volatile("griddepcontrol.wait;" ::: "memory");  // the partials of the attention kernel are complete
+  pdl_wait();  // the partials of the attention kernel are complete
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int bh = blockIdx.x; bh < BH; bh += gridDim.x) {
     const int2 r = ranges[bh];
@@ -443,24 +444,14 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   int levels = (int)(kMaxCtas / G);
   p.levels = levels > kLevels ? kLevels : (levels < 1 ? 1 : levels);
   p.scale_log2 = a.scale * kLog2e;
-  cross_attn_kernel<T, D><<<(unsigned)G, kThreads, smem, st>>>(p);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(cross_attn_kernel<T, D>, dim3((unsigned)G), dim3(kThreads), smem, st, p);
   if (e != cudaSuccess) return e;
-  // The merge as a programmatic dependent launch: it may be scheduled while
-  // the attention kernel drains and waits (griddepcontrol.wait) until that
-  // kernel has completed and its writes are visible.
+  // The merge, also a programmatic dependent: it may be scheduled while the
+  // attention kernel drains and waits (griddepcontrol.wait) until that kernel
+  // has completed and its writes are visible.
   const int BH = a.B * a.H;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(BH < 65535 ? BH : 65535));
-  cfg.blockDim = dim3(kMergeWarps * 32);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, cross_merge_kernel<D>, (const int2*)p.ranges, (const float*)p.partials, p.out, BH);
+  return launch_pdl(cross_merge_kernel<D>, dim3((unsigned)(BH < 65535 ? BH : 65535)), dim3(kMergeWarps * 32), 0, st,
+                    (const int2*)p.ranges, (const float*)p.partials, p.out, BH);
 }
 
 }  // namespace

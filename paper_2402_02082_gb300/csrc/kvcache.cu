@@ -19,6 +19,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "common.cuh"
 #include "kernels.h"
 
 namespace glide {
@@ -46,6 +47,7 @@ __global__ void __launch_bounds__(kThreads) kv_compact_kernel(const CompactParam
   constexpr int kRowBytes = RC * 16;
   constexpr int kPerLane = kBatch * RC / 32;  // chunks per lane and tensor per batch
   static_assert(kPerLane >= 1, "row too short");
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const long long slabs = (long long)p.layers * p.B * p.H;
   const long long warps = (long long)gridDim.x * kWarps;
@@ -141,13 +143,13 @@ cudaError_t launch_kv_compact(const CompactArgs& a, cudaStream_t st) {
   long long grid = (slabs + kWarps - 1) / kWarps;
   const long long cap = (long long)sm_count() * 8;
   if (grid > cap) grid = cap;
+  const dim3 g((unsigned)grid), blk(kThreads);
   switch (row_bytes / 16) {
-    case 8: kv_compact_kernel<8><<<(unsigned)grid, kThreads, 0, st>>>(p); break;
-    case 16: kv_compact_kernel<16><<<(unsigned)grid, kThreads, 0, st>>>(p); break;
-    case 32: kv_compact_kernel<32><<<(unsigned)grid, kThreads, 0, st>>>(p); break;
+    case 8: return launch_pdl(kv_compact_kernel<8>, g, blk, 0, st, p);
+    case 16: return launch_pdl(kv_compact_kernel<16>, g, blk, 0, st, p);
+    case 32: return launch_pdl(kv_compact_kernel<32>, g, blk, 0, st, p);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 }  // namespace glide

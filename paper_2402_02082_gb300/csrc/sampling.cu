@@ -69,6 +69,7 @@ __global__ void __launch_bounds__(kThreads) spec_sample_kernel(const SampleParam
   __shared__ float2 red[kWarps];
   __shared__ float seg_up[kWarps];
   __shared__ int last, s_tok, s_lastpos, s_win;
+  pdl_wait();
 
   const int G1 = p.gamma + 1;
   const int row = blockIdx.x;
@@ -267,8 +268,7 @@ cudaError_t launch_spec_sample(const SampleArgs& a, cudaStream_t st) {
   p.accept = reinterpret_cast<int*>(ws + off);
   const long long grid = (long long)a.B * (a.gamma + 1);
   if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
-  spec_sample_kernel<<<(unsigned)grid, kThreads, 0, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(spec_sample_kernel, dim3((unsigned)grid), dim3(kThreads), 0, st, p);
 }
 
 }  // namespace glide

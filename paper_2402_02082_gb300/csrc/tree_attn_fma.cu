@@ -68,6 +68,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_attn_fma_kernel(const TreePa
   using C = TreeCfg<T, D>;
   constexpr int E = C::E;
   constexpr int NS = C::NS;
+  pdl_wait();
   extern __shared__ __align__(1024) unsigned char smem[];
   T* sK = reinterpret_cast<T*>(smem + C::off_K);
   T* sV = reinterpret_cast<T*>(smem + C::off_V);
@@ -283,8 +284,7 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
   p.Hkv = a.Hkv; p.group = a.H / a.Hkv; p.rows = rows; p.R = R; p.tree = a.tree;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_fma_kernel<T, D><<<(unsigned)(G * R), kThreads, C::smem_bytes(a.B), st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(tree_attn_fma_kernel<T, D>, dim3((unsigned)(G * R)), dim3(kThreads), C::smem_bytes(a.B), st, p);
 }
 
 }  // namespace

@@ -192,6 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                         const TcParams p) {
   using C = TcCfg<D>;
+  pdl_wait();  // before any global access and before the TMEM allocation
   extern __shared__ unsigned char smem_raw[];
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int ns = p.ns;
@@ -714,8 +715,8 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.R = R; p.tree = a.tree;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  tree_attn_tc_kernel<D><<<(unsigned)(G * R), kThreads, C::smem_bytes(a.B, ns), st>>>(mk, mv, p);
-  return cudaGetLastError();
+  return launch_pdl(tree_attn_tc_kernel<D>, dim3((unsigned)(G * R)), dim3(kThreads), C::smem_bytes(a.B, ns), st,
+                    mk, mv, p);
 }
 
 }  // namespace
