@@ -770,8 +770,9 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
     # cached heads, D = 128), this workload's batch and context, the gamma = 5
     # chain of GliDe alone: one cross-attention call and one verification
     Hq, Hk, n6 = 32, 8, w.gamma + 1
+    n33 = 1 + CAPE_MAX_TOKENS   # a CaPE-sized tree: 132 query rows per cached head
     Lk = max(w.kv_len)
-    Sg = (Lk + n6 + 15) // 16 * 16
+    Sg = (Lk + n33 + 15) // 16 * 16
     gK = torch.randn(B, Hk, Sg, w.D, device=dev, dtype=torch.bfloat16)
     gV = torch.randn_like(gK)
     g_kv = torch.full((B,), Lk, dtype=torch.int32, device=dev)
@@ -780,10 +781,15 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
     g_par = torch.arange(-1, n6 - 1, dtype=torch.int32, device=dev).repeat(B, 1).contiguous()
     g_oc = torch.empty(B, 1, Hq, w.D, device=dev)
     g_ot = torch.empty(B, n6, Hq, w.D, device=dev)
-    g_ws = torch.zeros(gb.glide_attn_workspace_bytes(gb.make_desc(B, Hq, w.D, Sg, gb.GLIDE_BF16, H_kv=Hk), n6),
+    g_ws = torch.zeros(gb.glide_attn_workspace_bytes(gb.make_desc(B, Hq, w.D, Sg, gb.GLIDE_BF16, H_kv=Hk), n33),
                        dtype=torch.uint8, device=dev)
     gqa_c_ms = timed(lambda: gb.glide_cross_attn(g_qd, gK, gV, g_kv, Lk, g_oc, g_ws))
     gqa_t_ms = timed(lambda: gb.tree_verify_attn(g_qt, g_par, gK, gV, g_kv, Lk, g_ot, g_ws))
+    g_qt33 = torch.randn(B, n33, Hq, w.D, device=dev, dtype=torch.bfloat16)
+    g_par33 = torch.from_numpy(np.stack([synth.random_tree(w.seed + 40 + b, n33, 6, 5) for b in range(B)])).to(dev)
+    g_ot33 = torch.empty(B, n33, Hq, w.D, device=dev)
+    gqa_t33_ms = timed(lambda: gb.tree_verify_attn(g_qt33, g_par33, gK, gV, g_kv, Lk, g_ot33, g_ws))
+    gqa_t33_bytes = B * Hk * (Lk + n33) * w.D * 2 * 2 + B * n33 * Hq * w.D * (2 + 4) + 4 * B * (n33 + 1)
     gqa_c_bytes = B * Hk * Lk * w.D * 2 * 2 + B * Hq * w.D * (2 + 4)
     gqa_t_bytes = B * Hk * (Lk + n6) * w.D * 2 * 2 + B * n6 * Hq * w.D * (2 + 4) + 4 * B * (n6 + 1)
     del gK, gV
@@ -815,7 +821,10 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
             "cross_frac_of_peak": gqa_c_bytes / (gqa_c_ms * 1e-3) / 1e9 / peak,
             "verify_us": 1e3 * gqa_t_ms, "verify_gbs": gqa_t_bytes / (gqa_t_ms * 1e-3) / 1e9,
             "verify_frac_of_peak": gqa_t_bytes / (gqa_t_ms * 1e-3) / 1e9 / peak,
-            "shape": f"B={B} H=32 over H_kv=8 D={w.D} kv_len={Lk} bf16, chain of {n6} nodes"},
+            "verify_cape_us": 1e3 * gqa_t33_ms, "verify_cape_gbs": gqa_t33_bytes / (gqa_t33_ms * 1e-3) / 1e9,
+            "verify_cape_frac_of_peak": gqa_t33_bytes / (gqa_t33_ms * 1e-3) / 1e9 / peak,
+            "shape": f"B={B} H=32 over H_kv=8 D={w.D} kv_len={Lk} bf16, chain of {n6} nodes; "
+                     f"verify_cape: a random {n33}-node tree (CaPE's 32 verified tokens and the root)"},
         "spec_sample_accept": {"avg_us": 1e3 * samp_ms, "algo_bytes_per_launch": samp_bytes,
                                "achieved_gbs": samp_bytes / (samp_ms * 1e-3) / 1e9,
                                "frac_of_peak": samp_bytes / (samp_ms * 1e-3) / 1e9 / peak,
