@@ -240,138 +240,11 @@ __device__ inline void combine_if_last(const Segment& s, int H, int nq, int r0, 
   consumer_sync(nthreads);
 }
 
-// The arrival half of combine_if_last: after this CTA wrote its partial rows
-// for (b, h), count it in on counter cidx; returns true (in every calling
-// thread) if this CTA completed the count and so must merge the rows later
-// with combine_partials.  Called by all `nthreads` consumer threads.
-__device__ inline bool arrive_split(const Segment& s, int cidx, unsigned* counters, int ctid, int nthreads,
-                                    volatile int* flag) {
-  __threadfence();
-  consumer_sync(nthreads);
-  if (ctid == 0) {
-    const unsigned prev = atomicAdd(&counters[cidx], 1u);
-    *flag = (prev == (unsigned)(s.c_last - s.c_first)) ? 1 : 0;
-  }
-  consumer_sync(nthreads);
-  return *flag != 0;
-}
-
 // Where query row r of slab (b, h) goes in the output: out_row with nq / group
 // nodes (tree verification and grouped-query cross-attention).
 struct OutMap {
   int group, Hq;
   __device__ long long row(int b, int h, int r, int nq) const { return (long long)out_row(b, h, r, nq, group, Hq); }
 };
-
-// Merges rows [r0, r0 + nr) of every split partial of slab (b, h) =
-// (s.b, s.h) into `out` (query rows placed by the OutMap) and re-arms counter
-// cidx; all `nthreads` threads of the CTA call it (it uses __syncthreads).
-// scratch: shared memory for (2 + kCombineW) * nr floats.
-// Pass 1, one thread per query row: M = max_c m_c, the weights
-// w_c = 2^(m_c - M) and 1 / sum_c w_c l_c.  Pass 2: float4 outputs, each
-// thread taking kCombineU of them with every load issued before any use.
-constexpr int kCombineW = 8;   // slots whose weights are kept in shared memory
-constexpr int kCombineU = 3;   // outputs per thread per round
-__device__ inline void combine_partials(const Segment& s, int H, int nq, int r0, int nr, int cidx, int D,
-                                        const OutMap& om, const float* partials, unsigned* counters, float* out,
-                                        float* scratch, int tid, int nthreads) {
-  const int bh = s.b * H + s.h;
-  const int nsl = s.c_last - s.c_first + 1;
-  const int rs = D + 2;  // floats per partial row: m, l, o[D]
-  float* Mrow = scratch;
-  float* Linv = scratch + nr;
-  float* W = scratch + 2 * nr;
-  // row r0 of the first slot; consecutive CTAs' slots of one (b, h) are adjacent
-  const float* slot0 = partial_slot(const_cast<float*>(partials), s.c_first + bh, nq, D) + (size_t)r0 * rs;
-  const size_t sstride = (size_t)nq * rs;
-  __threadfence();
-  for (int r = tid; r < nr; r += nthreads) {
-    // one round of loads: (m, l) of every slot, with a running max
-    float M = -CUDART_INF_F, L = 0.f;
-#pragma unroll 4
-    for (int c = 0; c < nsl; ++c) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(slot0 + c * sstride + (size_t)r * rs));
-      if (ml.x > M) {
-        L = (M == -CUDART_INF_F ? 0.f : L * fast_exp2(M - ml.x)) + ml.y;
-        M = ml.x;
-      } else if (ml.x != -CUDART_INF_F) {
-        L += ml.y * fast_exp2(ml.x - M);
-      }
-      if (nsl <= kCombineW) W[r * kCombineW + c] = ml.x;
-    }
-    if (nsl <= kCombineW)
-      for (int c = 0; c < nsl; ++c) {
-        const float m = W[r * kCombineW + c];
-        W[r * kCombineW + c] = m == -CUDART_INF_F ? 0.f : fast_exp2(m - M);
-      }
-    Mrow[r] = M;
-    Linv[r] = L > 0.f ? 1.f / L : 0.f;
-  }
-  __syncthreads();
-  const int cpr = D / 4;
-  const int items = nr * cpr;
-  for (int base = tid; base < items; base += kCombineU * nthreads) {
-    float4 acc[kCombineU];
-#pragma unroll
-    for (int u = 0; u < kCombineU; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (nsl <= kCombineW) {
-      // slots in groups of 4: every load of a group is issued before any use
-      for (int c0 = 0; c0 < nsl; c0 += 4) {
-        float2 lo[kCombineU][4], hi[kCombineU][4];
-#pragma unroll
-        for (int u = 0; u < kCombineU; ++u) {
-          const int it = base + u * nthreads;
-          const int r = it / cpr, d0 = (it - r * cpr) * 4;
-#pragma unroll
-          for (int cc = 0; cc < 4; ++cc)
-            if (it < items && c0 + cc < nsl) {
-              const float* o = slot0 + (c0 + cc) * sstride + (size_t)r * rs + 2 + d0;
-              lo[u][cc] = __ldcg(reinterpret_cast<const float2*>(o));
-              hi[u][cc] = __ldcg(reinterpret_cast<const float2*>(o + 2));
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < kCombineU; ++u) {
-          const int it = base + u * nthreads;
-#pragma unroll
-          for (int cc = 0; cc < 4; ++cc)
-            if (it < items && c0 + cc < nsl) {
-              const float w = W[(it / cpr) * kCombineW + c0 + cc];
-              acc[u].x += w * lo[u][cc].x; acc[u].y += w * lo[u][cc].y;
-              acc[u].z += w * hi[u][cc].x; acc[u].w += w * hi[u][cc].y;
-            }
-        }
-      }
-    } else {
-      for (int c = 0; c < nsl; ++c) {
-#pragma unroll
-        for (int u = 0; u < kCombineU; ++u) {
-          const int it = base + u * nthreads;
-          if (it < items) {
-            const int r = it / cpr, d0 = (it - r * cpr) * 4;
-            const float* row = slot0 + c * sstride + (size_t)r * rs;
-            const float m = __ldcg(row);
-            const float w = m == -CUDART_INF_F ? 0.f : fast_exp2(m - Mrow[r]);
-            const float2 lo = __ldcg(reinterpret_cast<const float2*>(row + 2 + d0));
-            const float2 hi = __ldcg(reinterpret_cast<const float2*>(row + 4 + d0));
-            acc[u].x += w * lo.x; acc[u].y += w * lo.y; acc[u].z += w * hi.x; acc[u].w += w * hi.y;
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kCombineU; ++u) {
-      const int it = base + u * nthreads;
-      if (it < items) {
-        const int r = it / cpr, d0 = (it - r * cpr) * 4;
-        const float li = Linv[r];
-        *reinterpret_cast<float4*>(out + om.row(s.b, s.h, r0 + r, nq) * D + d0) =
-            make_float4(acc[u].x * li, acc[u].y * li, acc[u].z * li, acc[u].w * li);
-      }
-    }
-  }
-  if (tid == 0) counters[cidx] = 0u;
-  __syncthreads();
-}
 
 }  // namespace glide

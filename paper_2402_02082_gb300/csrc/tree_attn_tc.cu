@@ -47,6 +47,14 @@
 // sum taken with the same reference makes the result exact up to rounding.
 // V rows past the end of a slab are zeroed in shared memory before P.V (the
 // cache beyond kv_len + n may hold anything, even NaN).
+//
+// A slab whose keys fall in one CTA's share is written out directly.  A slab
+// split over several shares leaves one partial (max, sum, o) per share in the
+// workspace, and the kernel records the slab's share range; a second kernel,
+// tree_merge_kernel, launched as a programmatic dependent, merges them with
+// one warp per query row.  No CTA counts arrivals or merges at its end, so
+// the segment epilogues carry no fence or atomic and the merges run spread
+// over the whole GPU instead of on the last CTAs.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <math_constants.h>
@@ -109,7 +117,7 @@ struct TcParams {
   const int* parent;
   float* out;
   unsigned* status;
-  unsigned* counters;
+  int2* ranges;      // per slab: the share range of a split slab, (-1, -1) otherwise
   float* partials;
   int B, H, S_cap, max_kv_len, n;
   int Hkv;    // cached heads (slabs are (b, cached head))
@@ -201,9 +209,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   float2* ml = reinterpret_cast<float2*>(base + C::off_ml(ns));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + C::off_misc(ns));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 4);
-  volatile int* last_flag = reinterpret_cast<volatile int*>(base + C::off_misc(ns) + 8);
-  int* pend_count = reinterpret_cast<int*>(base + C::off_misc(ns) + 12);
-  int4* pend = reinterpret_cast<int4*>(base + C::off_misc(ns) + 16);  // at most 2 split segments
   BatchTiles bt;
   bt.start = reinterpret_cast<long long*>(base + C::off_tab(ns));
   bt.len = reinterpret_cast<int*>(bt.start + p.B + 1);
@@ -221,7 +226,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars[b], cnt);
     }
     *abort_flag = 0;
-    *pend_count = 0;
     fence_barrier_init();
   }
   if (warp == kMmaWarp) {
@@ -245,6 +249,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   Partition P;
   P.init(bt.start[p.B], gridDim.x / p.R);
   const long long g_begin = P.begin(x), g_end = P.end(x);
+  // The share range of every slab split over several shares, for the merge
+  // kernel ((-1, -1): written out directly, or no keys).
+  if (y == 0)
+    for (int bh = x * blockDim.x + threadIdx.x; bh < p.B * p.Hkv; bh += (gridDim.x / p.R) * blockDim.x) {
+      const int b = bh / p.Hkv, nt = bt.ntiles[b];
+      int2 r = make_int2(-1, -1);
+      if (nt > 0) {
+        const long long first = bt.start[b] + (long long)(bh - b * p.Hkv) * nt;
+        const int cf = P.cta_of(first), cl = P.cta_of(first + nt - 1);
+        if (cf != cl) r = make_int2(cf, cl);
+      }
+      p.ranges[bh] = r;
+    }
 
   if (warp == kProdWarp) {
     // ------------------------------------------------------------ producer
@@ -401,7 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int sid = threadIdx.x;                  // 0..255 among the softmax threads
     const float sl2 = p.scale_log2;
     bool dead = false;
-    int i = 0, seg = 0, npend = 0;
+    int i = 0, seg = 0;
     // Segment sg's queries into the swizzled Q tile (padding rows are zero);
     // the two threads of a row write chunks 0-3 and 4-7 of each 128-byte atom.
     // Key-half-0 warps only.
@@ -639,19 +656,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars[B_OFREE]);
-        // A split (b, h) is merged by the CTA that completes its count, but only
-        // after this CTA's last tile (see the end of the kernel), so that the
-        // merge does not hold up the next segment.  Only the first and the last
-        // segment of a CTA's share can be split.
-        if (!single && arrive_split(s, row_tile_counter(s.b, s.h, p.Hkv, p.R, y), p.counters, sid, kSoftWarps * 32,
-                                    last_flag)) {
-          if (sid == 0) pend[npend] = make_int4(s.b, s.h, s.c_first, s.c_last);
-          ++npend;
-        }
       }
       g = s.g_end;
     }
-    if (sid == 0) pend_count[0] = npend;
   }
 
   __syncwarp();  // the producer and MMA warps reconverge after their single-lane loops
@@ -661,16 +668,76 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, C::kTmemCols);
   }
-  // The split (b, h) this CTA completed, merged by all threads (no waiting,
-  // so also after an abort: the counters are re-armed either way); the P
-  // buffers, which no MMA reads any more, are the scratch.
-  const int np = pend_count[0];
-  for (int k = 0; k < np; ++k) {
-    Segment s;
-    s.b = pend[k].x; s.h = pend[k].y; s.c_first = pend[k].z; s.c_last = pend[k].w;
-    const OutMap om{p.group, p.H};
-    combine_partials(s, p.Hkv, p.rows, row0, rows_here, row_tile_counter(s.b, s.h, p.Hkv, p.R, y), D, om, p.partials,
-                     p.counters, p.out, reinterpret_cast<float*>(base + C::off_P), threadIdx.x, kThreads);
+}
+
+// Merges the partials of every split slab: one warp per query row r of slab
+// (b, cached head h) with share range [c_first, c_last] (ranges[bh]); the
+// partial of share c sits in slot c + bh, row r: [max, sum, o[D]] (log2
+// domain).  out = sum_c 2^(m_c - M) o_c / sum_c 2^(m_c - M) l_c, M = max_c m_c.
+// Each lane holds D / 32 columns (float2 pairs: a partial row is 8-byte
+// aligned); the loads of up to kMergeGroup shares are issued before any is
+// used, and groups fold into a running (max, sum, o).  A share whose max is
+// -inf (no visible key) has weight 0 and its o never reaches a sum.
+constexpr int kMergeGroup = 8;
+constexpr int kMergeWarps = 8;
+template <int D>
+__global__ void __launch_bounds__(kMergeWarps * 32) tree_merge_kernel(const int2* ranges, const float* partials,
+                                                                     float* out, int BH, int rows, int group, int Hq,
+                                                                     int Hkv) {
+  constexpr int kPairs = D / 64;  // float2 pairs per lane
+  pdl_wait();  // the partials and ranges of the verification kernel are complete
+  const int lane = threadIdx.x & 31;
+  const long long total = (long long)BH * rows;
+  for (long long wr = (long long)blockIdx.x * kMergeWarps + (threadIdx.x >> 5); wr < total;
+       wr += (long long)gridDim.x * kMergeWarps) {
+    const int bh = (int)(wr / rows), r = (int)(wr - (long long)bh * rows);
+    const int2 rg = ranges[bh];
+    if (rg.x < 0) continue;
+    const size_t sstride = (size_t)rows * (D + 2);
+    const float* row0 = partials + (size_t)(rg.x + bh) * sstride + (size_t)r * (D + 2);
+    const int nsl = rg.y - rg.x + 1;
+    float M = -CUDART_INF_F, L = 0.f;
+    float2 acc[kPairs];
+#pragma unroll
+    for (int k = 0; k < kPairs; ++k) acc[k] = make_float2(0.f, 0.f);
+    for (int c0 = 0; c0 < nsl; c0 += kMergeGroup) {
+      float2 ml[kMergeGroup], o[kMergeGroup][kPairs];
+#pragma unroll
+      for (int u = 0; u < kMergeGroup; ++u) {
+        const int c = c0 + u < nsl ? c0 + u : c0;
+        const float* pr = row0 + (size_t)c * sstride;
+        ml[u] = __ldcg(reinterpret_cast<const float2*>(pr));
+#pragma unroll
+        for (int k = 0; k < kPairs; ++k) o[u][k] = __ldcg(reinterpret_cast<const float2*>(pr + 2 + 64 * k + 2 * lane));
+        if (c0 + u >= nsl) ml[u].x = -CUDART_INF_F;
+      }
+      float Mg = M;
+#pragma unroll
+      for (int u = 0; u < kMergeGroup; ++u) Mg = fmaxf(Mg, ml[u].x);
+      if (Mg == -CUDART_INF_F) continue;
+      const float f = M == -CUDART_INF_F ? 0.f : fast_exp2(M - Mg);
+      L *= f;
+#pragma unroll
+      for (int k = 0; k < kPairs; ++k) acc[k] = make_float2(acc[k].x * f, acc[k].y * f);
+#pragma unroll
+      for (int u = 0; u < kMergeGroup; ++u) {
+        const bool live = ml[u].x != -CUDART_INF_F;
+        const float w = live ? fast_exp2(ml[u].x - Mg) : 0.f;
+        L += live ? w * ml[u].y : 0.f;
+#pragma unroll
+        for (int k = 0; k < kPairs; ++k) {
+          acc[k].x += live ? w * o[u][k].x : 0.f;  // a select: an unwritten o never reaches acc
+          acc[k].y += live ? w * o[u][k].y : 0.f;
+        }
+      }
+      M = Mg;
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    const int b = bh / Hkv, h = bh - b * Hkv;
+    float* dst = out + out_row(b, h, r, rows, group, Hq) * D;
+#pragma unroll
+    for (int k = 0; k < kPairs; ++k)
+      *reinterpret_cast<float2*>(dst + 64 * k + 2 * lane) = make_float2(acc[k].x * inv, acc[k].y * inv);
   }
 }
 
@@ -709,14 +776,21 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.out = a.out;
   unsigned char* ws = static_cast<unsigned char*>(a.ws);
   p.status = reinterpret_cast<unsigned*>(ws);
-  p.counters = reinterpret_cast<unsigned*>(ws + WsLayout::counters_off());
+  p.ranges = reinterpret_cast<int2*>(ws + WsLayout::ranges_off(a.B, a.H));
   p.partials = reinterpret_cast<float*>(ws + WsLayout::partials_off(a.B, a.H));
   p.B = a.B; p.H = a.H; p.S_cap = a.S_cap; p.max_kv_len = a.max_kv_len; p.n = a.nq;
   p.Hkv = a.Hkv; p.group = group; p.rows = p.n * group; p.R = R; p.tree = a.tree;
   p.ns = ns;
   p.scale_log2 = a.scale * kLog2e;
-  return launch_pdl(tree_attn_tc_kernel<D>, dim3((unsigned)(G * R)), dim3(kThreads), C::smem_bytes(a.B, ns), st,
-                    mk, mv, p);
+  cudaError_t e = launch_pdl(tree_attn_tc_kernel<D>, dim3((unsigned)(G * R)), dim3(kThreads), C::smem_bytes(a.B, ns),
+                             st, mk, mv, p);
+  if (e != cudaSuccess) return e;
+  // the merge of the split slabs: one warp per query row, at most four waves of CTAs over the SMs
+  const long long rows_total = (long long)a.B * a.Hkv * p.rows;
+  long long mg = (rows_total + kMergeWarps - 1) / kMergeWarps;
+  if (mg > 4LL * sm_count() * (2048 / (kMergeWarps * 32))) mg = 4LL * sm_count() * (2048 / (kMergeWarps * 32));
+  return launch_pdl(tree_merge_kernel<D>, dim3((unsigned)mg), dim3(kMergeWarps * 32), 0, st, (const int2*)p.ranges,
+                    (const float*)p.partials, p.out, a.B * a.Hkv, p.rows, group, a.H, a.Hkv);
 }
 
 }  // namespace
