@@ -265,6 +265,8 @@ constexpr int kMaxLevels = 6;
 constexpr long long kMinChunk = 16;
 struct Chunks {
   long long lo[kMaxLevels + 1];
+  long long base[kMaxLevels];  // tiles per chunk of level l (size / G) ...
+  int rem[kMaxLevels];         // ... and the first rem[l] chunks hold one more
   int G, L;
   __device__ void init(long long total, int grid, int levels) {
     G = grid;
@@ -274,29 +276,32 @@ struct Chunks {
       bool ok = true;
       for (int l = 0; l < L; ++l) {
         lo[l] = a;
-        const long long size = (l == L - 1) ? total - a : (total - a) / 2;
+        const long long size = (l == L - 1) ? total - a : (total - a) >> 1;
         if (size < G * kMinChunk) ok = false;
         a += size;
       }
       lo[L] = total;
       if (ok || L == 1) break;
     }
+    for (int l = 0; l < L; ++l) {  // the only divisions: once per level
+      const long long size = lo[l + 1] - lo[l];
+      base[l] = size / G;
+      rem[l] = (int)(size - base[l] * G);
+    }
   }
   __device__ int count() const { return G * L; }
   __device__ long long begin(int k) const {
     const int l = k / G, j = k - l * G;
     if (l >= L) return lo[L];
-    const long long size = lo[l + 1] - lo[l], base = size / G, rem = size % G;
-    return lo[l] + (long long)j * base + (j < rem ? j : rem);
+    return lo[l] + (long long)j * base[l] + (j < rem[l] ? j : rem[l]);
   }
   __device__ long long end(int k) const { return begin(k + 1); }
   __device__ int cta_of(long long g) const {
     int l = 0;
     while (l + 1 < L && g >= lo[l + 1]) ++l;
-    const long long size = lo[l + 1] - lo[l], base = size / G, rem = size % G;
     const long long off = g - lo[l];
-    const long long big = rem * (base + 1);
-    const long long j = off < big ? off / (base + 1) : rem + (off - big) / base;
+    const long long big = (long long)rem[l] * (base[l] + 1);
+    const long long j = off < big ? off / (base[l] + 1) : rem[l] + (off - big) / base[l];
     return l * G + (int)j;
   }
 };

@@ -10,9 +10,11 @@
 //   (Chunks) that the CTAs claim at run time: SMs do not all stream at the
 //   same rate, and a static equal split leaves the kernel waiting on the
 //   slowest ones;
-// * producer warp 0 claims the chunks (atomic counter in the workspace) and
-//   passes their ids to the other warps through a small shared-memory queue;
-//   all twelve warps walk the same chunk sequence;
+// * producer warp 0 claims the chunks (atomic counter in the workspace; a
+//   CTA's first chunk is its own block index, one of level 0's G chunks, so
+//   no claim delays the first copies) and passes their ids to the other warps
+//   through a small shared-memory queue; all twelve warps walk the same chunk
+//   sequence;
 // * four producer threads (one per producer warp; issuing a bulk copy keeps
 //   a thread busy for hundreds of cycles) stream K and V tiles with 1-D bulk
 //   copies (TMA) into shared-memory stages guarded by mbarriers; tile j of a
@@ -124,24 +126,6 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
   const Chunks& CK = s_chunks;
   const int nchunks = CK.count();
 
-  // The chunk range of every (b, h), for the merge kernel.
-  for (int bh = blockIdx.x * blockDim.x + threadIdx.x; bh < p.B * p.H; bh += gridDim.x * blockDim.x) {
-    const int b = bh / p.H, h = bh - b * p.H;
-    const int nt = bt.ntiles[b];
-    int2 r = make_int2(-1, -1);
-    if (nt > 0) {
-      const long long first = bt.start[b] + (long long)h * nt;
-      r = make_int2(CK.cta_of(first), CK.cta_of(first + nt - 1));
-    }
-    p.ranges[bh] = r;
-  }
-
-  // A sequence with no cached keys has an empty softmax: its output is zero.
-  for (int bh = blockIdx.x; bh < p.B * p.H; bh += gridDim.x) {
-    if (bt.ntiles[bh / p.H] == 0)
-      for (int d = threadIdx.x; d < D; d += blockDim.x) p.out[(size_t)bh * D + d] = 0.f;
-  }
-
   // The id of the q-th chunk this CTA works on (-1: no more work), read from
   // the queue by every warp but the claiming one.  Returns false on abort.
   auto next_chunk = [&](int q, int& k) -> bool {
@@ -174,7 +158,10 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
         if (pw == 0) {
           const int slot = q % kQN;
           if (!mbar_wait(&qempty[slot], ((q / kQN) & 1) ^ 1, abort_flag, p.status)) { ok = false; break; }
-          const unsigned c = atomicAdd(p.claim, 1u);
+          // The first chunk of CTA c is chunk c (the G chunks of level 0, one
+          // each: no atomic on the path to the first copy); later ones are
+          // claimed from the counter, which hands out chunks G, G + 1, ...
+          const unsigned c = q == 0 ? blockIdx.x : gridDim.x + atomicAdd(p.claim, 1u);
           k = c < (unsigned)nchunks ? (int)c : -1;
           qchunk[slot] = k;
           mbar_arrive(&qfull[slot]);
@@ -227,6 +214,25 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
   }
 
   // -------------------------------------------------------------- consumers
+  // The chunk range of every (b, h), for the merge kernel (written here, off
+  // the producers' path to their first copies).
+  for (int bh = blockIdx.x * (kNW * 32) + threadIdx.x; bh < p.B * p.H; bh += gridDim.x * (kNW * 32)) {
+    const int b = bh / p.H, h = bh - b * p.H;
+    const int nt = bt.ntiles[b];
+    int2 r = make_int2(-1, -1);
+    if (nt > 0) {
+      const long long first = bt.start[b] + (long long)h * nt;
+      r = make_int2(CK.cta_of(first), CK.cta_of(first + nt - 1));
+    }
+    p.ranges[bh] = r;
+  }
+
+  // A sequence with no cached keys has an empty softmax: its output is zero.
+  for (int bh = blockIdx.x; bh < p.B * p.H; bh += gridDim.x) {
+    if (bt.ntiles[bh / p.H] == 0)
+      for (int d = threadIdx.x; d < D; d += kNW * 32) p.out[(size_t)bh * D + d] = 0.f;
+  }
+
   const int sub = lane & 7, g4 = (lane >> 3) * 4;  // lane group g takes keys 4g..4g+3 of each tile
   const float sl2 = p.scale_log2;
   int uses = 0, q = 0;  // tiles this warp has taken from its ring so far
@@ -336,20 +342,21 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
 // Merges, for each (b, h), the partials of every consumer warp of every chunk
 // that holds part of its keys (slots (c + b*H + h) * 8 + w for c in its chunk
 // range): out = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s.  One CTA per
-// (b, h) (a (b, h) in the small late chunks has a few hundred partials):
-// threads stride over the partials for M and the sum, then each of the 16
-// warps takes every 16th partial, lanes owning D / 32 consecutive columns,
-// with a group of 8 partials' loads issued before any use; the warps' sums
-// meet in shared memory.  A warp that had no tile of a segment left max = -inf and no o: its
-// weight is 0 and its o never reaches a sum.
+// (b, h): warp w takes partials w, w + 16, ..., the loads of up to
+// kMergeGroup of them issued together (one round of loads for a (b, h) with
+// up to 128 partials), each lane holding D / 32 columns as float2 pairs (a
+// partial row is 8-byte aligned), and folds them into a running (max, sum, o);
+// the 16 warps' results meet in shared memory.  A partial whose max is -inf
+// (a warp that had no tile of the segment) has weight 0 and its o never
+// reaches a sum.
 constexpr int kMergeWarps = 16;
 constexpr int kMergeGroup = 8;  // partials per warp whose loads are issued together
 template <int D>
 __global__ void __launch_bounds__(kMergeWarps * 32) cross_merge_kernel(const int2* ranges, const float* partials,
                                                                       float* out, int BH) {
-  constexpr int kCols = D / 32;
+  constexpr int kPairs = D / 64;
   __shared__ float red[kMergeWarps][D];
-  __shared__ float stat[2][kMergeWarps];
+  __shared__ float2 stat[kMergeWarps];
   pdl_wait();  // the partials of the attention kernel are complete
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int bh = blockIdx.x; bh < BH; bh += gridDim.x) {
@@ -357,58 +364,60 @@ __global__ void __launch_bounds__(kMergeWarps * 32) cross_merge_kernel(const int
     if (r.x < 0) continue;  // a sequence with no cached keys: the attention kernel wrote zeros
     const int nsl = kNW * (r.y - r.x + 1);
     const float* base = partials + (size_t)(r.x + bh) * kNW * (D + 2);  // the slots are adjacent
-    float M = -CUDART_INF_F;
-    for (int q = threadIdx.x; q < nsl; q += blockDim.x) M = fmaxf(M, __ldcg(base + (size_t)q * (D + 2)));
-    M = warp_max(M);
-    if (lane == 0) stat[0][warp] = M;
-    __syncthreads();
-    M = stat[0][0];
+    float M = -CUDART_INF_F, L = 0.f;
+    float2 acc[kPairs];
 #pragma unroll
-    for (int w = 1; w < kMergeWarps; ++w) M = fmaxf(M, stat[0][w]);
-    float Ls = 0.f;
-    for (int q = threadIdx.x; q < nsl; q += blockDim.x) {
-      const float2 ml = __ldcg(reinterpret_cast<const float2*>(base + (size_t)q * (D + 2)));
-      if (ml.x != -CUDART_INF_F) Ls += fast_exp2(ml.x - M) * ml.y;
-    }
-    Ls = warp_sum(Ls);
-    if (lane == 0) stat[1][warp] = Ls;
-    float acc[kCols];
-#pragma unroll
-    for (int c = 0; c < kCols; ++c) acc[c] = 0.f;
+    for (int k = 0; k < kPairs; ++k) acc[k] = make_float2(0.f, 0.f);
     for (int q0 = warp; q0 < nsl; q0 += kMergeWarps * kMergeGroup) {
-      float mq[kMergeGroup];
-      float2 o[kMergeGroup][kCols / 2];
+      float2 ml[kMergeGroup], o[kMergeGroup][kPairs];
 #pragma unroll
       for (int u = 0; u < kMergeGroup; ++u) {
         const int qq = q0 + u * kMergeWarps;
-        const int q = qq < nsl ? qq : warp;
-        const float* row = base + (size_t)q * (D + 2);
-        mq[u] = qq < nsl ? __ldcg(row) : -CUDART_INF_F;
+        const float* row = base + (size_t)(qq < nsl ? qq : q0) * (D + 2);
+        ml[u] = __ldcg(reinterpret_cast<const float2*>(row));
 #pragma unroll
-        for (int c = 0; c < kCols / 2; ++c) o[u][c] = __ldcg(reinterpret_cast<const float2*>(row + 2 + lane * kCols) + c);
+        for (int k = 0; k < kPairs; ++k) o[u][k] = __ldcg(reinterpret_cast<const float2*>(row + 2 + 64 * k + 2 * lane));
+        if (qq >= nsl) ml[u].x = -CUDART_INF_F;
       }
+      float Mg = M;
+#pragma unroll
+      for (int u = 0; u < kMergeGroup; ++u) Mg = fmaxf(Mg, ml[u].x);
+      if (Mg == -CUDART_INF_F) continue;
+      const float f = M == -CUDART_INF_F ? 0.f : fast_exp2(M - Mg);
+      L *= f;
+#pragma unroll
+      for (int k = 0; k < kPairs; ++k) acc[k] = make_float2(acc[k].x * f, acc[k].y * f);
 #pragma unroll
       for (int u = 0; u < kMergeGroup; ++u) {
-        const bool live = mq[u] != -CUDART_INF_F;
-        const float w = live ? fast_exp2(mq[u] - M) : 0.f;
+        const bool live = ml[u].x != -CUDART_INF_F;
+        const float w = live ? fast_exp2(ml[u].x - Mg) : 0.f;
+        L += live ? w * ml[u].y : 0.f;
 #pragma unroll
-        for (int c = 0; c < kCols / 2; ++c) {
-          acc[2 * c] += live ? w * o[u][c].x : 0.f;   // a select: an unwritten o never reaches acc
-          acc[2 * c + 1] += live ? w * o[u][c].y : 0.f;
+        for (int k = 0; k < kPairs; ++k) {
+          acc[k].x += live ? w * o[u][k].x : 0.f;  // a select: an unwritten o never reaches acc
+          acc[k].y += live ? w * o[u][k].y : 0.f;
         }
       }
+      M = Mg;
     }
+    if (lane == 0) stat[warp] = make_float2(M, L);
 #pragma unroll
-    for (int c = 0; c < kCols; ++c) red[warp][lane * kCols + c] = acc[c];
+    for (int k = 0; k < kPairs; ++k) *reinterpret_cast<float2*>(&red[warp][64 * k + 2 * lane]) = acc[k];
     __syncthreads();
-    float L = 0.f;
+    float Mt = -CUDART_INF_F;
 #pragma unroll
-    for (int w = 0; w < kMergeWarps; ++w) L += stat[1][w];
-    const float li = L > 0.f ? 1.f / L : 0.f;
+    for (int w = 0; w < kMergeWarps; ++w) Mt = fmaxf(Mt, stat[w].x);
+    float Lt = 0.f, wt[kMergeWarps];
+#pragma unroll
+    for (int w = 0; w < kMergeWarps; ++w) {
+      wt[w] = stat[w].x == -CUDART_INF_F ? 0.f : fast_exp2(stat[w].x - Mt);
+      Lt += wt[w] * stat[w].y;
+    }
+    const float li = Lt > 0.f ? 1.f / Lt : 0.f;
     for (int d = threadIdx.x; d < D; d += blockDim.x) {
       float v = 0.f;
 #pragma unroll
-      for (int w = 0; w < kMergeWarps; ++w) v += red[w][d];
+      for (int w = 0; w < kMergeWarps; ++w) v += wt[w] * red[w][d];
       out[(size_t)bh * D + d] = v * li;
     }
     __syncthreads();

@@ -234,12 +234,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc::fence_before_sync();
   build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? n : 0, kTK);  // __syncthreads inside
-  if (!p.tree) {  // prefix only: a sequence with no cached keys has an empty softmax, output zero
-    const long long total = (long long)p.B * n * p.H * D;
-    for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-         idx += (long long)gridDim.x * blockDim.x)
-      if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
-  }
   tc::fence_after_sync();
   const uint32_t tmem = *tmem_slot;
 
@@ -249,19 +243,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   Partition P;
   P.init(bt.start[p.B], gridDim.x / p.R);
   const long long g_begin = P.begin(x), g_end = P.end(x);
-  // The share range of every slab split over several shares, for the merge
-  // kernel ((-1, -1): written out directly, or no keys).
-  if (y == 0)
-    for (int bh = x * blockDim.x + threadIdx.x; bh < p.B * p.Hkv; bh += (gridDim.x / p.R) * blockDim.x) {
-      const int b = bh / p.Hkv, nt = bt.ntiles[b];
-      int2 r = make_int2(-1, -1);
-      if (nt > 0) {
-        const long long first = bt.start[b] + (long long)(bh - b * p.Hkv) * nt;
-        const int cf = P.cta_of(first), cl = P.cta_of(first + nt - 1);
-        if (cf != cl) r = make_int2(cf, cl);
-      }
-      p.ranges[bh] = r;
-    }
 
   if (warp == kProdWarp) {
     // ------------------------------------------------------------ producer
@@ -403,6 +384,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------- softmax
+    // Off the producer's path to its first loads: the share range of every
+    // slab split over several shares, for the merge kernel ((-1, -1): written
+    // out directly, or no keys), and zeros for a prefix-only call's sequences
+    // without cached keys (an empty softmax).
+    constexpr int kST = kSoftWarps * 32;
+    if (y == 0)
+      for (int bh = x * kST + (int)threadIdx.x; bh < p.B * p.Hkv; bh += (gridDim.x / p.R) * kST) {
+        const int b = bh / p.Hkv, nt = bt.ntiles[b];
+        int2 r = make_int2(-1, -1);
+        if (nt > 0) {
+          const long long first = bt.start[b] + (long long)(bh - b * p.Hkv) * nt;
+          const int cf = P.cta_of(first), cl = P.cta_of(first + nt - 1);
+          if (cf != cl) r = make_int2(cf, cl);
+        }
+        p.ranges[bh] = r;
+      }
+    if (!p.tree) {
+      const long long total = (long long)p.B * n * p.H * D;
+      for (long long idx = (long long)blockIdx.x * kST + threadIdx.x; idx < total; idx += (long long)gridDim.x * kST)
+        if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
+    }
     // Warp w reads lane quarter q = w % 4 (MMA rows 16q..16q+15) and key half
     // w / 4 with the 16x64b TMEM shape: lane pair (t, t^2) shares one row,
     // thread t takes the row's even or odd columns (cpar), 16 of the 32 keys.
