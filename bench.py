@@ -926,6 +926,23 @@ def run_glide(args, rank, world, local_rank):
     value = job_throughput(step_kv * args.steps, world, elapsed_ms * 1e-3) / 1e9
     tree_tok = job_throughput(B * n * args.steps, world, elapsed_ms * 1e-3)
 
+    # ---- the acceptance's cost inside the round: [verify, accept] minus [verify]
+    # back to back (events around a single short launch also time the event
+    # machinery, ~2 us steps on this GPU, and break the programmatic launch
+    # chain between the two calls)
+    pairs_va, pairs_v = [], []
+    for _ in range(max(10, args.steps // 4)):
+        for lst, fns in ((pairs_va, step_fns[-2:]), (pairs_v, step_fns[-2:-1])):
+            a, b = event_pair()
+            a.record(stream)
+            for f in fns:
+                f()
+            b.record(stream)
+            lst.append((a, b))
+    torch.cuda.synchronize()
+    accept_marginal_ms = (statistics.mean(a.elapsed_time(b) for a, b in pairs_va) -
+                          statistics.mean(a.elapsed_time(b) for a, b in pairs_v))
+
     # ---- end to end: per-round inputs from pinned host memory, results back to host
     e2e_steps = max(3, min(args.steps, args.e2e_steps))
     e2e_eager_s, e2e_graph_s, e2e_launch = time_e2e(r.e2e_enqueue, dev, e2e_steps, world)
@@ -948,6 +965,11 @@ def run_glide(args, rank, world, local_rank):
         kernels[nm] = {"avg_us": 1e3 * avg_ms, "launches_per_step": names.count(nm),
                        "share": names.count(nm) * avg_ms * args.steps / sum(sum(v) for v in per_kernel.values()),
                        "algo_bytes_per_launch": ab[nm], "achieved_gbs": ach, "frac_of_peak": ach / peak}
+    acc_b = ab["tree_accept"]
+    kernels["tree_accept"]["in_round"] = {
+        "marginal_us": 1e3 * accept_marginal_ms, "achieved_gbs": acc_b / (accept_marginal_ms * 1e-3) / 1e9,
+        "frac_of_peak": acc_b / (accept_marginal_ms * 1e-3) / 1e9 / peak,
+        "how": "mean of [tree_verify_attn, tree_accept] minus mean of [tree_verify_attn], back to back"}
     dom = max(kernels, key=lambda k: kernels[k]["share"])
     roof = {"kernel": dom, "bound": "hbm", "achieved": kernels[dom]["achieved_gbs"], "peak": peak,
             "peak_source": peak_src, "unit": "GB/s", "frac": kernels[dom]["frac_of_peak"],

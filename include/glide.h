@@ -106,7 +106,8 @@ typedef struct {
   int32_t H_kv;       /* cached (key/value) heads; 0 means H.  H % H_kv == 0: each run of
                          H / H_kv consecutive query heads shares one cached head (grouped-
                          query attention, as in Mistral-7B: 32 query over 8 cached heads).
-                         tree_verify_attn needs n * H / H_kv <= 64.                       */
+                         tree_verify_attn needs n * H / H_kv <= 256 (query rows per
+                         cached head; more than 64 are served in row tiles of 64).        */
 } glide_attn_desc;
 
 /* Version of this ABI (GLIDE_ABI_VERSION of the built library). */
