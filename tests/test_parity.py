@@ -275,3 +275,72 @@ def test_accept_ties_and_signed_zero():
     want = oracle.tree_accept(toks, parents, lg)
     assert list(got[0][0]) == list(want[0][0]) == [0, 1, 2] and got[1][0] == want[1][0] == 2
     assert got[2][0] == want[2][0] == 0
+
+
+def test_accept_many_chunks_per_warp():
+    """300 sequences of 64 nodes over 16384 logits: 76800 chunks of 4096
+    logits on 152 CTAs of 14 consumer warps, so every warp counts more than a
+    full batch of 32 chunks and some warps complete several sequences in one
+    batch."""
+    parents, toks, lg = accept_case(300, 64, 16384, seed=777, p=0.8)
+    got = run_accept(parents, toks, lg)
+    want = oracle.tree_accept(toks, parents, lg)
+    for gv, wv in zip(got, want):
+        assert np.array_equal(gv, wv)
+
+
+def test_accept_ties_across_chunks_and_infinite_rows():
+    """Equal maxima in different 4096-logit chunks of a row go to the lowest
+    index, -0 equals +0 across chunks, a maximum in a row's ragged last chunk
+    is found, and a row of -inf has its argmax at 0 (as numpy's)."""
+    V = 32000
+    lg = np.random.default_rng(5).standard_normal((2, 4, V)).astype(np.float32)
+    lg[0, 0, [20000, 100, 31999]] = 9.0            # ties in chunks 4, 0 and 7 -> 100
+    lg[0, 1, :] = -1.0
+    lg[0, 1, [12288 + 5, 4096 * 7 + 3]] = 0.0      # +0 in chunk 3 ...
+    lg[0, 1, 8191] = -0.0                           # ... -0 in chunk 1 wins by index
+    lg[0, 2, 31999] = 50.0                          # the last logit of the ragged chunk
+    lg[0, 3, :] = -np.inf
+    lg[1] = lg[0, ::-1]
+    parents = np.array([[-1, 0, 1, 2]] * 2, dtype=np.int32)
+    a = oracle.row_argmax(lg)
+    toks = np.stack([np.r_[0, a[b, :3]] for b in range(2)]).astype(np.int32)   # every edge matches
+    got = run_accept(parents, toks, lg)
+    want = oracle.tree_accept(toks, parents, lg)
+    assert list(a[0]) == [100, 8191, 31999, 0]
+    for gv, wv in zip(got, want):
+        assert np.array_equal(gv, wv)
+    assert list(got[1]) == [3, 3] and list(got[2]) == [0, 100]
+
+
+def test_accept_invalid_parents_are_safe():
+    """Parent arrays that break the contract (out of range, a second root,
+    a parent after its child) give meaningless but well-formed results: no
+    fault, a clean workspace, and a path that is a chain of matched edges
+    from node 0 to a deepest node whose whole parent chain is valid and
+    matched (the documented rule: a parent outside [0, c) makes node c
+    unreachable)."""
+    g = np.random.default_rng(31)
+    B, n, V = 6, 64, 1000
+    parents, toks, lg = accept_case(B, n, V, seed=4242, p=0.9)
+    for b in range(B):
+        for c in range(1, n):
+            if g.random() < 0.12:
+                parents[b, c] = int(g.choice([-1, -5, c, c + 3, n + 7, 2 ** 30]))
+    path, ln, bonus = run_accept(parents, toks, lg)
+    a = oracle.row_argmax(lg)
+    for b in range(B):
+        def chain(c):   # the root path of c, or None when it leaves [0, c) or an edge does not match
+            out = [c]
+            while c != 0:
+                p = int(parents[b, c])
+                if not (0 <= p < c) or toks[b, c] != a[b, p]:
+                    return None
+                out.append(p)
+                c = p
+            return out[::-1]
+        ok = {c: chain(c) for c in range(n)}
+        best = max((len(v) - 1, -c) for c, v in ok.items() if v is not None)
+        node = -best[1]
+        assert ln[b] == best[0] and bonus[b] == a[b, node]
+        assert list(path[b, :ln[b] + 1]) == ok[node] and all(path[b, ln[b] + 1:] == -1)
