@@ -20,7 +20,7 @@
 // together and stream the same K/V tiles at about the same time: DRAM serves
 // each tile about once and L2 the other R - 1 reads.
 //
-// Roles (384 threads, persistent grid of one CTA per SM, split-KV partition
+// Roles (416 threads, persistent grid of one CTA per SM, split-KV partition
 // shared with the other attention kernels):
 //   warps 0-7  softmax.  An M = 64 accumulator keeps rows 16q..16q+15 in
 //              TMEM lanes 32q..32q+15; warp w reads lane quarter q = w % 4
@@ -31,10 +31,10 @@
 //              the halves are merged once per segment.  Query i sits in row
 //              (i % 4) * 16 + i / 4, which spreads any tree over all four lane
 //              quarters (all four SM sub-partitions).
-//   warp 8     producer: lane 0 feeds both the K and the V ring with 2-D TMA
-//              (64 keys x 64 head dims per box, 128-byte swizzle), polling
-//              both rings' free slots without blocking on either (K slots free
-//              up after S, V slots only after P.V).
+//   warps 8, 12 producers: lane 0 of warp 8 feeds the K ring, lane 0 of
+//              warp 12 the V ring, with 2-D TMA (64 keys x 64 head dims per
+//              box, 128-byte swizzle); K slots free up after S, V slots only
+//              after P.V, so each ring has its own thread.
 //   warps 9-11 MMA issue.  A tcgen05.mma keeps its issuing thread busy for
 //              ~150 cycles whatever its shape, so one thread cannot feed a
 //              64-key tile (8 S + 4 P.V instructions) at HBM speed: warp 9
@@ -73,9 +73,10 @@ constexpr int kM = 64;           // MMA rows (tree queries, zero-padded)
 constexpr int kMaxStages = 8;    // K/V stages (the launch picks as many as fit)
 constexpr int kSBuf = 4;         // S buffers in TMEM (two per S issuer)
 constexpr int kSoftWarps = 8;
-constexpr int kProdWarp = 8;
+constexpr int kProdWarp = 8;     // the K ring's producer
 constexpr int kMmaWarp = 9;      // warps 9, 10: S issuers; warp 11: P.V issuer
-constexpr int kThreads = 384;
+constexpr int kVProdWarp = 12;   // the V ring's producer
+constexpr int kThreads = 416;
 constexpr float kRescaleLog2 = 8.0f;
 
 // barrier slots
@@ -244,77 +245,41 @@ __global__ void __launch_bounds__(kThreads, 1)
   P.init(bt.start[p.B], gridDim.x / p.R);
   const long long g_begin = P.begin(x), g_end = P.end(x);
 
-  if (warp == kProdWarp) {
-    // ------------------------------------------------------------ producer
-    // One thread feeds both rings without blocking on either: K slots free up
-    // when S is done, V slots only when P.V is done, and a blocking wait on
-    // one ring would hold back the other.
+  if (warp == kProdWarp || warp == kVProdWarp) {
+    // ----------------------------------------------------------- producers
+    // Warp 8 feeds the K ring and warp 12 the V ring, one thread each: a
+    // 2-D tensor copy keeps its issuing thread busy for hundreds of cycles,
+    // and one thread issuing both rings' copies (four per 64-key tile) set
+    // the pace of the whole kernel at ~1430 cycles per tile (per-tile trace:
+    // each copy left 1.3-1.9 tile periods after its slot was free).
     if (lane == 0) {
-      tc::prefetch_tmap(&tmK);
-      tc::prefetch_tmap(&tmV);
+      const bool is_k = warp == kProdWarp;
+      const CUtensorMap* map = is_k ? &tmK : &tmV;
+      tc::prefetch_tmap(map);
+      uint64_t* full = &bars[is_k ? B_KFULL : B_VFULL];
+      uint64_t* empty = &bars[is_k ? B_KEMPTY : B_VEMPTY];
+      const uint32_t dst0 = is_k ? C::off_K : off_V;
       // one reader per tile: evict it first; R row tiles read each tile R times
       const uint64_t pol = p.R == 1 ? policy_evict_first() : policy_evict_normal();
-      struct Cursor {  // next tile to load: CTA-local index i, segment s, tile t
-        int i, t;
-        long long g;
-        Segment s;
-      };
-      auto start_seg = [&](Cursor& c) {
-        if (c.g < g_end) {
-          c.s = locate(bt, P, p.B, c.g, g_end);
-          c.t = c.s.t0;
+      int i = 0;
+      bool ok = true;
+      for (long long g = g_begin; g < g_end && ok;) {
+        const Segment sg = locate(bt, P, p.B, g, g_end);
+        const int row0k = (sg.b * p.Hkv + sg.h) * p.S_cap;
+        for (int t = sg.t0; t < sg.t1; ++t, ++i) {
+          const int st = i % ns;
+          if (!mbar_wait(&empty[st], ((i / ns) & 1) ^ 1, abort_flag, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[st], C::kKVTile);
+          for (int hd = 0; hd < C::kHalves; ++hd)
+            tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, row0k + t * kTK, &full[st],
+                            pol);
         }
-      };
-      auto issue = [&](Cursor& c, const CUtensorMap* map, uint64_t* full, uint32_t dst0) {
-        const int st = c.i % ns;
-        mbar_arrive_expect_tx(&full[st], C::kKVTile);
-        const int row = (c.s.b * p.Hkv + c.s.h) * p.S_cap + c.t * kTK;
-        for (int hd = 0; hd < C::kHalves; ++hd)
-          tc::tma_load_2d(base + dst0 + st * C::kKVTile + hd * C::kKVHalf, map, hd * 64, row, &full[st], pol);
-        ++c.i;
-        if (++c.t == c.s.t1) {
-          c.g = c.s.g_end;
-          start_seg(c);
-        }
-      };
-      Cursor ck, cv;
-      ck.i = cv.i = 0;
-      ck.g = cv.g = g_begin;
-      start_seg(ck);
-      start_seg(cv);
-      const int total = (int)(g_end - g_begin);
-      uint64_t t_last = global_timer_ns();
-      int spins = 0, seen = 0;
-      while (ck.i < total || cv.i < total) {
-        bool progressed = false;
-        if (ck.i < total && mbar_test_wait(&bars[B_KEMPTY + ck.i % ns], ((ck.i / ns) & 1) ^ 1)) {
-          issue(ck, &tmK, &bars[B_KFULL], C::off_K);
-          progressed = true;
-        }
-        if (cv.i < total && mbar_test_wait(&bars[B_VEMPTY + cv.i % ns], ((cv.i / ns) & 1) ^ 1)) {
-          issue(cv, &tmV, &bars[B_VFULL], off_V);
-          progressed = true;
-        }
-        if (progressed || ++spins < 64) continue;
-        spins = 0;  // every 64 idle polls: check for an abort or a stall of more than kWaitLimitNs
-        const uint64_t now = global_timer_ns();
-        if (ck.i + cv.i != seen) {
-          seen = ck.i + cv.i;
-          t_last = now;
-        }
-        if (*abort_flag) break;
-        if (now - t_last > kWaitLimitNs) {
-          *abort_flag = 1;
-          record_status(p.status, kStatusTimeout);
-          break;
-        }
+        g = sg.g_end;
       }
-      if (ck.i < total || cv.i < total) {  // aborted: let issued loads land before the CTA exits
-        for (int j = (ck.i > ns ? ck.i - ns : 0); j < ck.i; ++j) mbar_drain(&bars[B_KFULL + j % ns], (j / ns) & 1);
-        for (int j = (cv.i > ns ? cv.i - ns : 0); j < cv.i; ++j) mbar_drain(&bars[B_VFULL + j % ns], (j / ns) & 1);
-      }
+      if (!ok)  // aborted: let issued loads land before the CTA exits
+        for (int j = (i > ns ? i - ns : 0); j < i; ++j) mbar_drain(&full[j % ns], (j / ns) & 1);
     }
-  } else if (warp >= kMmaWarp) {
+  } else if (warp >= kMmaWarp) {  // warps 9-11
     // ----------------------------------------------------------- MMA issue
     const int role = warp - kMmaWarp;  // 0, 1: S of tiles with j % 2 == role; 2: P.V
     if (lane == 0) {
