@@ -20,6 +20,7 @@ import argparse
 import dataclasses
 import hashlib
 import json
+import math
 import multiprocessing as mp
 import os
 import statistics
@@ -476,6 +477,27 @@ def time_e2e(enqueue, dev, steps, world):
         return eager_s, None, f"eager (graph capture failed: {type(exc).__name__})"
 
 
+def time_back_to_back(fns, reps, flush=None, lead_ms=4.0):
+    """Average CUDA-event time (ms) of one call in a run of `reps` calls issued
+    back to back on the current stream (call i is fns[i % len(fns)]), the
+    way a serving loop issues them.  A GPU-side wait of about lead_ms runs
+    first, so the host has enqueued every call before the first one starts:
+    the run times the device, not the host's launch rate, and one event pair
+    spans all the calls.  With `flush` the L2 is evicted before the run."""
+    import torch
+    stream = torch.cuda.current_stream()
+    if flush is not None:
+        flush()
+    torch.cuda._sleep(int(lead_ms * 2.0e6))   # clock cycles at ~2 GHz
+    a, b = event_pair()
+    a.record(stream)
+    for i in range(reps):
+        fns[i % len(fns)]()
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
 def time_steps_events(step, steps, flush=None):
     """CUDA-event time (ms) of each of `steps` calls of step() on the current
     stream; with `flush` (an L2Flush), the L2 is evicted before every step
@@ -808,7 +830,25 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
     gqa_t33_bytes = B * Hk * (Lk + n33) * w.D * 2 * 2 + B * n33 * Hq * w.D * (2 + 4) + 4 * B * (n33 + 1)
     gqa_c_bytes = B * Hk * Lk * w.D * 2 * 2 + B * Hq * w.D * (2 + 4)
     gqa_t_bytes = B * Hk * (Lk + n6) * w.D * 2 * 2 + B * n6 * Hq * w.D * (2 + 4) + 4 * B * (n6 + 1)
-    del gK, gV
+    # the same calls over the caches of eight layers in turn, back to back, as
+    # a verification pass over a target model's layers issues them (each
+    # layer's cache is its own, so every call reads its K/V from HBM)
+    n_lay = 8
+    lay = [(gK, gV)] + [(torch.randn_like(gK), torch.randn_like(gV)) for _ in range(n_lay - 1)]
+    gqa_layers = {}
+    for nm, mk, nb in (("cross", lambda k, v: lambda: gb.glide_cross_attn(g_qd, k, v, g_kv, Lk, g_oc, g_ws), gqa_c_bytes),
+                       ("verify", lambda k, v: lambda: gb.tree_verify_attn(g_qt, g_par, k, v, g_kv, Lk, g_ot, g_ws),
+                        gqa_t_bytes),
+                       ("verify_cape", lambda k, v: lambda: gb.tree_verify_attn(g_qt33, g_par33, k, v, g_kv, Lk, g_ot33,
+                                                                                g_ws), gqa_t33_bytes)):
+        fns = [mk(k, v) for k, v in lay]
+        ms = statistics.median(time_back_to_back(fns, 4 * n_lay) for _ in range(3))
+        gqa_layers[nm + "_us"] = 1e3 * ms
+        gqa_layers[nm + "_gbs"] = nb / (ms * 1e-3) / 1e9
+        gqa_layers[nm + "_frac_of_peak"] = nb / (ms * 1e-3) / 1e9 / peak
+    gqa_layers["how"] = (f"{n_lay} layers' caches in turn, {4 * n_lay} calls back to back, one event pair "
+                         "around the run (mean call duration)")
+    del lay, gK, gV
     # the draft's training-time cross-attention under the block mask (L = 5) on a
     # Vicuna-7B training shape: B = 4 sequences of T = 2048, 32 heads, D = 128
     Bt, Tt, Ht, Lb = 4, 2048, 32, 5
@@ -839,6 +879,7 @@ def time_next_rows(args, w, case, gb, dev, stream, K, V, kv_len, peak):
             "verify_frac_of_peak": gqa_t_bytes / (gqa_t_ms * 1e-3) / 1e9 / peak,
             "verify_cape_us": 1e3 * gqa_t33_ms, "verify_cape_gbs": gqa_t33_bytes / (gqa_t33_ms * 1e-3) / 1e9,
             "verify_cape_frac_of_peak": gqa_t33_bytes / (gqa_t33_ms * 1e-3) / 1e9 / peak,
+            "layers_back_to_back": gqa_layers,
             "shape": f"B={B} H=32 over H_kv=8 D={w.D} kv_len={Lk} bf16, chain of {n6} nodes; "
                      f"verify_cape: a random {n33}-node tree (CaPE's 32 verified tokens and the root)"},
         "spec_sample_accept": {"avg_us": 1e3 * samp_ms, "algo_bytes_per_launch": samp_bytes,
@@ -935,6 +976,26 @@ def run_glide(args, rank, world, local_rank):
     if not r.status_ok():
         raise RuntimeError("device status not OK after the per-call timing")
 
+    # ---- each call back to back (the per-call durations of the roofline and
+    # the shares): events around a single short launch also time the event
+    # machinery (~2 us steps on this GPU) and the launch itself.  The K/V
+    # caches are far larger than L2; the logits rows of tree_accept are not,
+    # so its calls rotate over enough copies of them (> 2 x L2) that every
+    # call reads its logits from HBM.
+    import torch
+    g = w.gamma
+    n_acc = max(2, int(math.ceil(2 * L2_BYTES / max(1, r.logits.numel() * 4))))
+    acc_logits = [r.logits] + [r.logits.clone() for _ in range(n_acc - 1)]
+    acc_fns = [lambda lg=lg: gb.tree_accept(r.draft, r.parent, lg, r.path, r.ln, r.bonus, r.ws_acc)
+               for lg in acc_logits]
+    b2b_ms = {}
+    for nm, fns, reps in (("glide_cross_attn", step_fns[:g], 2 * g), ("tree_verify_attn", step_fns[g:g + 1], 8),
+                          ("tree_accept", acc_fns, 64)):
+        b2b_ms[nm] = statistics.median(time_back_to_back(fns, reps) for _ in range(3))
+    del acc_logits, acc_fns
+    if not r.status_ok():
+        raise RuntimeError("device status not OK after the back-to-back timing")
+
     step_kv = r.kv_bytes_per_step()
     value = job_throughput(step_kv * args.steps, world, elapsed_ms * 1e-3) / 1e9
     tree_tok = job_throughput(B * n * args.steps, world, elapsed_ms * 1e-3)
@@ -972,12 +1033,15 @@ def run_glide(args, rank, world, local_rank):
     # ---- roofline of the dominant kernel
     ab = algo_bytes(w)
     kernels = {}
+    tot_ms = sum(names.count(k) * v for k, v in b2b_ms.items())
     for nm, times in per_kernel.items():
-        avg_ms = sum(times) / len(times)
+        avg_ms = b2b_ms[nm]
         ach = ab[nm] / (avg_ms * 1e-3) / 1e9
         kernels[nm] = {"avg_us": 1e3 * avg_ms, "launches_per_step": names.count(nm),
-                       "share": names.count(nm) * avg_ms * args.steps / sum(sum(v) for v in per_kernel.values()),
-                       "algo_bytes_per_launch": ab[nm], "achieved_gbs": ach, "frac_of_peak": ach / peak}
+                       "share": names.count(nm) * avg_ms / tot_ms,
+                       "algo_bytes_per_launch": ab[nm], "achieved_gbs": ach, "frac_of_peak": ach / peak,
+                       "how": "mean call duration in a run of back-to-back calls, one event pair around the run",
+                       "alone_us": 1e3 * sum(times) / len(times)}
     acc_b = ab["tree_accept"]
     kernels["tree_accept"]["in_round"] = {
         "marginal_us": 1e3 * accept_marginal_ms, "achieved_gbs": acc_b / (accept_marginal_ms * 1e-3) / 1e9,

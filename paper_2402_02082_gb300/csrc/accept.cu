@@ -9,9 +9,10 @@
 //    CTA's chunks with 1-D bulk copies (TMA) into a ring of kNS shared-memory
 //    stages, so nearly all of the logits are in flight at once; stage s always
 //    serves consumer warp s, which reduces the whole chunk (a float max over
-//    each lane's float4 groups, the index recovered from the winning group,
-//    then a warp reduction) and folds one 64-bit key (order-preserving float
-//    bits above the complemented index) into the row's slot with atomicMax.
+//    each lane's float4 groups, loaded eight at a time into eight independent
+//    chains, the index recovered from the winning group, then two redux
+//    max reductions of a 64-bit key: order-preserving float bits above the
+//    complemented index) and folds the key into the row's slot with atomicMax.
 //    The logits are a plain HBM stream.
 // 2. every chunk is counted into its sequence's counter (release fence, then
 //    an acquire atomic; nothing waits).  The warp that completes a sequence's
@@ -71,24 +72,73 @@ __device__ __forceinline__ int key_index(unsigned long long k) {
 }
 
 // Counter increment with acquire semantics: a thread that sees the final
-// count also sees every slot update fenced before the other increments.
+// count also sees every slot update released before the other increments.
 __device__ __forceinline__ unsigned atomic_add_acquire(unsigned* addr, unsigned v) {
   unsigned old;
   asm volatile("atom.acquire.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(addr), "r"(v) : "memory");
   return old;
 }
 
-// (value, index) pairs: the larger value wins, the lower index among equals.
-__device__ __forceinline__ void warp_argmax(float& m, int& idx) {
+// The warp's largest key (every lane gets it): two max reductions, the high
+// words first, then the low words of the lanes that hold the largest high word.
+__device__ __forceinline__ unsigned long long warp_max_key(unsigned long long k) {
+  const uint32_t hi = (uint32_t)(k >> 32), lo = (uint32_t)k;
+  const uint32_t mhi = __reduce_max_sync(0xffffffffu, hi);
+  const uint32_t mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? lo : 0u);
+  return ((unsigned long long)mhi << 32) | mlo;
+}
+
+// Release fence at GPU scope: the writes before it (and those seen through
+// a warp barrier) are visible before any write after it.
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+
+// One lane's part of a chunk in shared memory: the float4 groups lane,
+// lane + 32, ... below n4 (all kGroups of them when kFull).  Groups are loaded
+// eight at a time into eight independent chains (group i goes to chain
+// i % 8); a strict comparison keeps the first group of each chain holding the
+// chain's maximum, and the chains are combined lowest group first among equal
+// maxima.  Returns the lane's maximum and the group holding its first
+// occurrence (-1 when the lane has no group).
+template <bool kFull>
+__device__ __forceinline__ int scan_lane(const float4* s4, int n4, int lane, float& best) {
+  constexpr int kC = 8;
+  float acc[kC];
+  int grp[kC];
 #pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) {
-    const float om = __shfl_xor_sync(0xffffffffu, m, off);
-    const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
-    if (om > m || (om == m && oi < idx)) {
-      m = om;
-      idx = oi;
+  for (int j = 0; j < kC; ++j) {
+    acc[j] = -__int_as_float(0x7f800000);
+    grp[j] = -1;
+  }
+#pragma unroll
+  for (int b = 0; b < kGroups / kC; ++b) {
+    float4 v[kC];
+#pragma unroll
+    for (int j = 0; j < kC; ++j) {
+      const int q = lane + 32 * (b * kC + j);
+      if (kFull || q < n4) v[j] = s4[q];
+    }
+#pragma unroll
+    for (int j = 0; j < kC; ++j) {
+      const int q = lane + 32 * (b * kC + j);
+      if (kFull || q < n4) {
+        const float g = fmaxf(fmaxf(v[j].x, v[j].y), fmaxf(v[j].z, v[j].w));
+        if (b == 0 || grp[j] < 0 || g > acc[j]) {
+          acc[j] = g;
+          grp[j] = b * kC + j;
+        }
+      }
     }
   }
+  float m = acc[0];
+  int gi = grp[0];
+#pragma unroll
+  for (int j = 1; j < kC; ++j)
+    if (grp[j] >= 0 && (gi < 0 || acc[j] > m || (acc[j] == m && grp[j] < gi))) {
+      m = acc[j];
+      gi = grp[j];
+    }
+  best = m;
+  return gi;
 }
 
 // Value of node `c`'s copy of a per-node quantity held two nodes per lane
@@ -247,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
   int pend_seq = 0, npend = 0;  // lane i: the sequence of the warp's i-th uncounted chunk
   auto count_in = [&]() {
     __syncwarp();
-    __threadfence();  // the warp's slot updates are visible before any of its counts
+    fence_acq_rel_gpu();  // release: the warp's slot updates are visible before any of its counts
     const bool mine = lane < npend;
     unsigned prev = 0;
     if (mine) prev = atomic_add_acquire(&p.counters[pend_seq], 1u);
@@ -272,46 +322,9 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
       if (!mbar_wait(&full[warp], (uint32_t)(use & 1), abort_flag, p.status)) break;
       const float4* s4 = reinterpret_cast<const float4*>(ring + (size_t)warp * kChunk);
       const int n4 = cnt >> 2;  // cnt is a multiple of 4 in this mode
-      // The lane's float4 groups in increasing index order, even and odd groups
-      // in two independent chains; a strict comparison keeps the first group
-      // holding each chain's maximum, and the index inside it comes after.
-      float ma = m, mb = m;
-      int ga = -1, gb = -1;
-      if (lane < n4) {
-        const float4 v = s4[lane];
-        ma = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
-        ga = 0;
-      }
-      if (lane + 32 < n4) {
-        const float4 v = s4[lane + 32];
-        mb = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
-        gb = 1;
-      }
-#pragma unroll 4
-      for (int i = 2; i < kGroups; i += 2) {
-        const int q = lane + 32 * i;
-        if (q < n4) {
-          const float4 v = s4[q];
-          const float g = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
-          if (g > ma) {
-            ma = g;
-            ga = i;
-          }
-        }
-        if (q + 32 < n4) {
-          const float4 v = s4[q + 32];
-          const float g = fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w));
-          if (g > mb) {
-            mb = g;
-            gb = i + 1;
-          }
-        }
-      }
-      if (gb >= 0 && (mb > ma || (mb == ma && gb < ga))) {
-        ma = mb;
-        ga = gb;
-      }
-      if (ga >= 0) {
+      float ma;
+      const int ga = n4 == kChunk / 4 ? scan_lane<true>(s4, n4, lane, ma) : scan_lane<false>(s4, n4, lane, ma);
+      if (ga >= 0) {  // the index inside the winning group
         const float4 v = s4[lane + 32 * ga];
         const int e = v.x == ma ? 0 : (v.y == ma ? 1 : (v.z == ma ? 2 : 3));
         m = ma;
@@ -333,8 +346,8 @@ __global__ void __launch_bounds__(kThreads, 1) tree_accept_kernel(const AccParam
         }
       }
     }
-    warp_argmax(m, idx);
-    if (lane == 0) atomicMax(&p.slots[row], argmax_key(m, idx));
+    const unsigned long long key = warp_max_key(argmax_key(m, idx));
+    if (lane == 0) atomicMax(&p.slots[row], key);
     if (lane == npend) pend_seq = (int)(row / p.n);
     if (++npend == 32) count_in();
   }
