@@ -268,25 +268,29 @@ struct Chunks {
   long long base[kMaxLevels];  // tiles per chunk of level l (size / G) ...
   int rem[kMaxLevels];         // ... and the first rem[l] chunks hold one more
   int G, L;
-  __device__ void init(long long total, int grid, int levels) {
-    G = grid;
-    L = levels < 1 ? 1 : (levels > kMaxLevels ? kMaxLevels : levels);
-    for (;; --L) {
-      long long a = 0;
-      bool ok = true;
-      for (int l = 0; l < L; ++l) {
-        lo[l] = a;
-        const long long size = (l == L - 1) ? total - a : (total - a) >> 1;
-        if (size < G * kMinChunk) ok = false;
-        a += size;
-      }
-      lo[L] = total;
-      if (ok || L == 1) break;
+  // Built by lanes 0 .. kMaxLevels - 1 of one warp together (every lane of
+  // that warp must call).  Level l's remainder r_l = total - lo[l] is
+  // ceil(total / 2^l) (l halvings with the ceiling are one shift), and level
+  // sizes never grow from one level to the next, so the levels that fit are a
+  // prefix that one ballot counts; each lane then fills its own level, and the
+  // per-level divisions run side by side.
+  __device__ void init_warp(long long total, int grid, int levels, int lane) {
+    const int Lmax = levels < 1 ? 1 : (levels > kMaxLevels ? kMaxLevels : levels);
+    const int l = lane < kMaxLevels ? lane : kMaxLevels - 1;
+    const long long r = (total + (1ll << l) - 1) >> l;
+    // L levels fit when level L - 2 (the smallest halved one) holds G * kMinChunk tiles
+    const bool fits = lane <= Lmax - 2 && (r >> 1) >= (long long)grid * kMinChunk;
+    const int nl = 1 + __popc(__ballot_sync(0xffffffffu, fits));
+    if (lane < nl) {
+      lo[lane] = total - r;
+      const long long size = lane == nl - 1 ? r : (r >> 1);
+      base[lane] = size / grid;
+      rem[lane] = (int)(size - base[lane] * grid);
     }
-    for (int l = 0; l < L; ++l) {  // the only divisions: once per level
-      const long long size = lo[l + 1] - lo[l];
-      base[l] = size / G;
-      rem[l] = (int)(size - base[l] * G);
+    if (lane == 0) {
+      lo[nl] = total;
+      G = grid;
+      L = nl;
     }
   }
   __device__ int count() const { return G * L; }

@@ -89,7 +89,6 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
   using C = CrossCfg<T, D>;
   using G = GroupMap<T, D>;
   constexpr int NS = C::NS;
-  pdl_wait();
   extern __shared__ __align__(1024) unsigned char smem[];
   T* sK = reinterpret_cast<T*>(smem + C::off_K);
   T* sV = reinterpret_cast<T*>(smem + C::off_V);
@@ -118,10 +117,11 @@ __global__ void __launch_bounds__(kThreads, 1) cross_attn_kernel(const CrossPara
     *abort_flag = 0;
     fence_barrier_init();
   }
+  pdl_wait();  // shared-memory set-up above; every global access below
   build_batch_tiles(bt, p.kv_len, p.B, p.H, p.max_kv_len, 0, kTK);  // ends with __syncthreads
 
   __shared__ Chunks s_chunks;  // one copy of the level table, not one per thread
-  if (threadIdx.x == 0) s_chunks.init(bt.start[p.B], gridDim.x, p.levels);
+  if (warp == 0) s_chunks.init_warp(bt.start[p.B], gridDim.x, p.levels, lane);
   __syncthreads();
   const Chunks& CK = s_chunks;
   const int nchunks = CK.count();

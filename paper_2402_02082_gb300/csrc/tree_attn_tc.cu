@@ -201,7 +201,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                         const TcParams p) {
   using C = TcCfg<D>;
-  pdl_wait();  // before any global access and before the TMEM allocation
   extern __shared__ unsigned char smem_raw[];
   unsigned char* base = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int ns = p.ns;
@@ -218,7 +217,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = p.n;
+  // Shared-memory set-up and the tensor-map fetches (kernel parameters) come
+  // before the wait for the previous kernel; every global access and the TMEM
+  // allocation come after it.
   if (threadIdx.x == 0) {
+    tc::prefetch_tmap(&tmK);
+    tc::prefetch_tmap(&tmV);
     for (int b = 0; b < kNumBars; ++b) {
       uint32_t cnt = 1;
       if ((b >= B_SFREE && b < B_SFREE + kSBuf) || b == B_PFULL || b == B_PFULL + 1) cnt = kSoftWarps;
@@ -229,6 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
+  pdl_wait();
   if (warp == kMmaWarp) {
     tc::tmem_alloc(tmem_slot, C::kTmemCols);
     tc::tmem_relinquish();
