@@ -354,27 +354,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------- softmax
-    // Off the producer's path to its first loads: the share range of every
-    // slab split over several shares, for the merge kernel ((-1, -1): written
-    // out directly, or no keys), and zeros for a prefix-only call's sequences
-    // without cached keys (an empty softmax).
-    constexpr int kST = kSoftWarps * 32;
-    if (y == 0)
-      for (int bh = x * kST + (int)threadIdx.x; bh < p.B * p.Hkv; bh += (gridDim.x / p.R) * kST) {
-        const int b = bh / p.Hkv, nt = bt.ntiles[b];
-        int2 r = make_int2(-1, -1);
-        if (nt > 0) {
-          const long long first = bt.start[b] + (long long)(bh - b * p.Hkv) * nt;
-          const int cf = P.cta_of(first), cl = P.cta_of(first + nt - 1);
-          if (cf != cl) r = make_int2(cf, cl);
-        }
-        p.ranges[bh] = r;
-      }
-    if (!p.tree) {
-      const long long total = (long long)p.B * n * p.H * D;
-      for (long long idx = (long long)blockIdx.x * kST + threadIdx.x; idx < total; idx += (long long)gridDim.x * kST)
-        if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
-    }
     // Warp w reads lane quarter q = w % 4 (MMA rows 16q..16q+15) and key half
     // w / 4 with the 16x64b TMEM shape: lane pair (t, t^2) shares one row,
     // thread t takes the row's even or odd columns (cpar), 16 of the 32 keys.
@@ -420,15 +399,39 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars[B_QFULL + (sg & 1)]);
     };
+    // The first segment's queries first: the first S products wait for them.
+    if (half == 0 && g_begin < g_end) write_q(locate(bt, P, p.B, g_begin, g_end), 0);
+    // Then, off the path to the first S products: the share range of every
+    // slab split over several shares, for the merge kernel ((-1, -1): written
+    // out directly, or no keys), and zeros for a prefix-only call's sequences
+    // without cached keys (an empty softmax).
+    constexpr int kST = kSoftWarps * 32;
+    if (y == 0)
+      for (int bh = x * kST + (int)threadIdx.x; bh < p.B * p.Hkv; bh += (gridDim.x / p.R) * kST) {
+        const int b = bh / p.Hkv, nt = bt.ntiles[b];
+        int2 r = make_int2(-1, -1);
+        if (nt > 0) {
+          const long long first = bt.start[b] + (long long)(bh - b * p.Hkv) * nt;
+          const int cf = P.cta_of(first), cl = P.cta_of(first + nt - 1);
+          if (cf != cl) r = make_int2(cf, cl);
+        }
+        p.ranges[bh] = r;
+      }
+    if (!p.tree) {
+      const long long total = (long long)p.B * n * p.H * D;
+      for (long long idx = (long long)blockIdx.x * kST + threadIdx.x; idx < total; idx += (long long)gridDim.x * kST)
+        if (bt.ntiles[idx / ((long long)n * p.H * D)] == 0) p.out[idx] = 0.f;
+    }
     for (long long g = g_begin; g < g_end; ++seg) {
       const Segment s = locate(bt, P, p.B, g, g_end);
       const int plen = bt.plen[s.b], len = bt.len[s.b];
       int rowlim;  // keys below it are visible to this row (the prefix)
       const long long orow = row_at(s, rowlim);
 
-      if (half == 0 && seg == 0) write_q(s, 0);  // later segments' Q is written ahead (below)
-      uint64_t anc = 0;  // ancestor-or-self set of this row's tree node
-      if (p.tree) anc = ancestors(p.parent + (size_t)s.b * n, n, node, valid, lane);  // prefix only: no tree keys
+      // the ancestor-or-self set of this row's tree node, found when the first
+      // tile with tree keys comes (prefix only: no tree keys)
+      uint64_t anc = 0;
+      bool anc_ready = !p.tree;
 
       float m_used = -CUDART_INF_F, l = 0.f;  // l: this thread's share of the row sum
       // S of the next tile is loaded while this tile's exponentials run (within
@@ -459,6 +462,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 16; ++k) sc[k] = __uint_as_float(cur[k]) * sl2;
         } else {
+          if (!anc_ready) {  // warp-uniform: t, half and plen are the same in every lane
+            anc = ancestors(p.parent + (size_t)s.b * n, n, node, valid, lane);
+            anc_ready = true;
+          }
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
             const int key = key0 + 2 * k;
