@@ -78,6 +78,13 @@ constexpr int kMmaWarp = 9;      // warps 9, 10: S issuers; warp 11: P.V issuer
 constexpr int kVProdWarp = 12;   // the V ring's producer
 constexpr int kThreads = 416;
 constexpr float kRescaleLog2 = 8.0f;
+// What a switch from one slab to the next costs a CTA, in 64-key tiles: per
+// CTA, the end times of a static split grow by ~2.7 us per extra segment at 4
+// query rows, ~5 us at 24 and ~5.5 us at 64 (the epilogue of one slab, with
+// its output or partial rows, and the pipeline start of the next) at ~0.7 us
+// per tile, so shares are balanced on tiles + w * (segments - 1) with
+// w = 4 + rows / 16.
+__host__ __device__ constexpr int seg_weight(int rows) { return 4 + rows / 16; }
 
 // barrier slots
 // ODONE has four slots (tile mod 4): the softmax waits on it only now and
@@ -109,7 +116,7 @@ struct TcCfg {
   static constexpr uint32_t kTmemCols = kTmemO + 2 * D <= 256 ? 256 : 512;
   static_assert(kTmemO + 2 * D <= 512, "TMEM columns");
   static_assert(kNumBars * 8 <= 512, "barrier area");
-  static size_t smem_bytes(int B, int ns) { return 1024 + off_tab(ns) + (size_t)(B + 1) * 8 + (size_t)3 * B * 4; }
+  static size_t smem_bytes(int B, int ns) { return 1024 + off_tab(ns) + (size_t)(B + 1) * 8 + (size_t)(4 * B + 1) * 4; }
 };
 
 struct TcParams {
@@ -214,6 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   bt.len = reinterpret_cast<int*>(bt.start + p.B + 1);
   bt.ntiles = bt.len + p.B;
   bt.plen = bt.ntiles + p.B;
+  bt.sidx = bt.plen + p.B;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = p.n;
@@ -246,8 +254,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // this CTA: share x of the key sequence, row tile y of every slab in it
   const int x = blockIdx.x / p.R, y = blockIdx.x - x * p.R;
   const int row0 = y * kM, rows_here = min(kM, p.rows - row0);
-  Partition P;
-  P.init(bt.start[p.B], gridDim.x / p.R);
+  CostPartition P;  // shares of equal cost, a segment switch counted as seg_weight tiles
+  P.init(bt, p.B, p.Hkv, gridDim.x / p.R, seg_weight(p.rows < kM ? p.rows : kM));
   const long long g_begin = P.begin(x), g_end = P.end(x);
 
   if (warp == kProdWarp || warp == kVProdWarp) {
