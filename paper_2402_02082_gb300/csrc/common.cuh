@@ -68,11 +68,14 @@ __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w &
 // tail.  pdl_wait() blocks until the previous grid has completed and its
 // writes are visible; a kernel calls it before its first global-memory access
 // and before it allocates tensor memory, so it never reads an input early nor
-// holds resources the previous grid could wait for.  No kernel signals its
-// dependents early (griddepcontrol.launch_dependents): measured, dependents
-// resident next to a running kernel slowed it (one round of the 7B chain
-// workload: 115 us without the early signal, 128 us with it, 142 us with no
-// programmatic launch at all).
+// holds resources the previous grid could wait for.  Only the two split-merge
+// kernels signal their dependents early (griddepcontrol.launch_dependents, at
+// their start): the next attention kernel's CTAs are then placed on the SMs
+// the small merge grid leaves free and wait there, so its launch overlaps the
+// merge (batch-1 Vicuna-7B round 93.8 -> 91.5 us).  An early signal from the
+// attention kernels, which fill every SM, slowed them instead (dependents
+// resident next to a running kernel: one 7B chain round 115 us without the
+// signal, 128 us with it in every kernel, 142 us with no programmatic launch).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 template <typename... KArgs, typename... Args>

@@ -357,6 +357,9 @@ __global__ void __launch_bounds__(kMergeWarps * 32) cross_merge_kernel(const int
   constexpr int kPairs = D / 64;
   __shared__ float red[kMergeWarps][D];
   __shared__ float2 stat[kMergeWarps];
+  // The next kernel may be scheduled now, onto the SMs this small grid leaves
+  // free; it waits for this merge to complete before it touches memory.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   pdl_wait();  // the partials of the attention kernel are complete
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int bh = blockIdx.x; bh < BH; bh += gridDim.x) {

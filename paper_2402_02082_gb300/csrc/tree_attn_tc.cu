@@ -672,6 +672,9 @@ __global__ void __launch_bounds__(kMergeWarps * 32) tree_merge_kernel(const int2
                                                                      float* out, int BH, int rows, int group, int Hq,
                                                                      int Hkv) {
   constexpr int kPairs = D / 64;  // float2 pairs per lane
+  // The next kernel may be scheduled now, onto the SMs this small grid leaves
+  // free; it waits for this merge to complete before it touches memory.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   pdl_wait();  // the partials and ranges of the verification kernel are complete
   const int lane = threadIdx.x & 31;
   const long long total = (long long)BH * rows;
