@@ -267,56 +267,56 @@ __device__ inline void build_batch_tiles(BatchTiles bt, const int* kv_len, int B
 // about the same time.  Tile g of the s-th slab with tiles sits at position
 // g + w * s of a cost line [0, C), C = tiles + w * (slabs - 1); the line is
 // split into G equal parts (sizes differ by at most one) and a share holds
-// the tiles whose positions fall in its part.  Needs bt.sidx.
+// the tiles whose positions fall in its part.  Needs bt.sidx.  The caller
+// keeps tiles + w * slabs below 2^31, so the arithmetic is 32-bit.
 struct CostPartition {
   BatchTiles bt;
-  int B, G;
-  int H;
-  long long w, C, base, rem, T;
+  int B, G, H, w, C, base, rem, T;
   __device__ void init(const BatchTiles& t, int nb, int nh, int grid, int weight) {
     bt = t;
     B = nb;
     H = nh;
     G = grid;
     w = weight;
-    T = bt.start[B];
-    const long long S = bt.sidx[B];
+    T = (int)bt.start[B];
+    const int S = bt.sidx[B];
     C = T + (S > 0 ? w * (S - 1) : 0);
     base = C / G;
     rem = C - base * G;
   }
   // position of the first tile of sequence b, if b has tiles
-  __device__ long long seq_pos(int b) const { return bt.start[b] + w * bt.sidx[b]; }
-  __device__ long long part_begin(int c) const { return (long long)c * base + (c < rem ? c : rem); }
+  __device__ int seq_pos(int b) const { return (int)bt.start[b] + w * bt.sidx[b]; }
+  __device__ int part_begin(int c) const { return c * base + (c < rem ? c : rem); }
   // the first tile at a position >= v (T if none)
-  __device__ long long tile_at(long long v) const {
+  __device__ long long tile_at(int v) const {
     if (v >= C) return T;
     int lo = 0, hi = B - 1;  // last b with seq_pos(b) <= v: a sequence with tiles
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
       if (seq_pos(mid) <= v) lo = mid; else hi = mid - 1;
     }
-    const long long nt = bt.ntiles[lo];
-    const long long off = v - seq_pos(lo);
-    long long h = nt > 0 ? off / (nt + w) : 0;
+    const int nt = bt.ntiles[lo];
+    const int off = v - seq_pos(lo);
+    int h = nt > 0 ? off / (nt + w) : 0;
     if (h > H - 1) h = H - 1;
-    const long long r = off - h * (nt + w);
-    const long long g0 = bt.start[lo] + h * nt;
+    const int r = off - h * (nt + w);
+    const int g0 = (int)bt.start[lo] + h * nt;
     return r < nt ? g0 + r : g0 + nt;  // a position between two slabs: the next slab's first tile
   }
   __device__ long long begin(int c) const { return tile_at(part_begin(c)); }
   __device__ long long end(int c) const { return tile_at(part_begin(c + 1)); }
-  __device__ int cta_of(long long g) const {
+  __device__ int cta_of(long long g64) const {
+    const int g = (int)g64;
     int lo = 0, hi = B - 1;  // the sequence of tile g
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (bt.start[mid] <= g) lo = mid; else hi = mid - 1;
+      if ((int)bt.start[mid] <= g) lo = mid; else hi = mid - 1;
     }
-    const long long h = (g - bt.start[lo]) / bt.ntiles[lo];
-    const long long v = g + w * (bt.sidx[lo] + h);
-    const long long big = rem * (base + 1);
-    if (v < big || base == 0) return (int)(v / (base + 1));
-    return (int)(rem + (v - big) / base);
+    const int h = (g - (int)bt.start[lo]) / bt.ntiles[lo];
+    const int v = g + w * (bt.sidx[lo] + h);
+    const int big = rem * (base + 1);
+    if (v < big || base == 0) return v / (base + 1);
+    return rem + (v - big) / base;
   }
 };
 
