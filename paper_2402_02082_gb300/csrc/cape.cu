@@ -39,7 +39,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kTop = 8;          // the proposal token + at most 7 expansion tokens
-constexpr int kChunk = 4096;     // probabilities per CTA
+constexpr int kChunk = 2048;     // probabilities per CTA (8 a thread: shorter insertion chains than 16)
 constexpr int kPerThread = kChunk / kThreads;
 static_assert(kPerThread % 4 == 0, "a thread's share is whole float4s");
 constexpr int kMaxPos = kMaxTree - 1;  // gamma <= max_tokens <= 63
