@@ -268,11 +268,12 @@ __device__ inline void build_batch_tiles(BatchTiles bt, const int* kv_len, int B
 // g + w * s of a cost line [0, C), C = tiles + w * (slabs - 1); the line is
 // split into G equal parts (sizes differ by at most one) and a share holds
 // the tiles whose positions fall in its part.  Needs bt.sidx.  The caller
-// keeps tiles + w * slabs below 2^31, so the arithmetic is 32-bit.
+// keeps tiles + w * slabs below 2^31, so the arithmetic is 32-bit.  Plain
+// arithmetic on the table only, so the host can check it too.
 struct CostPartition {
   BatchTiles bt;
   int B, G, H, w, C, base, rem, T;
-  __device__ void init(const BatchTiles& t, int nb, int nh, int grid, int weight) {
+  __host__ __device__ void init(const BatchTiles& t, int nb, int nh, int grid, int weight) {
     bt = t;
     B = nb;
     H = nh;
@@ -285,10 +286,10 @@ struct CostPartition {
     rem = C - base * G;
   }
   // position of the first tile of sequence b, if b has tiles
-  __device__ int seq_pos(int b) const { return (int)bt.start[b] + w * bt.sidx[b]; }
-  __device__ int part_begin(int c) const { return c * base + (c < rem ? c : rem); }
+  __host__ __device__ int seq_pos(int b) const { return (int)bt.start[b] + w * bt.sidx[b]; }
+  __host__ __device__ int part_begin(int c) const { return c * base + (c < rem ? c : rem); }
   // the first tile at a position >= v (T if none)
-  __device__ long long tile_at(int v) const {
+  __host__ __device__ long long tile_at(int v) const {
     if (v >= C) return T;
     int lo = 0, hi = B - 1;  // last b with seq_pos(b) <= v: a sequence with tiles
     while (lo < hi) {
@@ -303,9 +304,9 @@ struct CostPartition {
     const int g0 = (int)bt.start[lo] + h * nt;
     return r < nt ? g0 + r : g0 + nt;  // a position between two slabs: the next slab's first tile
   }
-  __device__ long long begin(int c) const { return tile_at(part_begin(c)); }
-  __device__ long long end(int c) const { return tile_at(part_begin(c + 1)); }
-  __device__ int cta_of(long long g64) const {
+  __host__ __device__ long long begin(int c) const { return tile_at(part_begin(c)); }
+  __host__ __device__ long long end(int c) const { return tile_at(part_begin(c + 1)); }
+  __host__ __device__ int cta_of(long long g64) const {
     const int g = (int)g64;
     int lo = 0, hi = B - 1;  // the sequence of tile g
     while (lo < hi) {
