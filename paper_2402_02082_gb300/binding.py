@@ -26,6 +26,7 @@ GLIDE_ERR_DEVICE_TIMEOUT = 4
 GLIDE_BF16 = 0
 GLIDE_F32 = 1
 GLIDE_FLAG_FORCE_FMA = 1
+GLIDE_FLAG_TILE64 = 2
 
 
 class GlideError(RuntimeError):

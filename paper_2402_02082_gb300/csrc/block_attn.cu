@@ -67,6 +67,7 @@
 
 #include "attn_common.cuh"
 #include "kernels.h"
+#include "tc_attn.cuh"
 #include "tc_ptx.cuh"
 #include "tensor_map.h"
 
@@ -204,56 +205,6 @@ struct Walker {
 };
 
 
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-// Warp-uniform bounded wait: every lane probes once and the warp votes; only
-// if the phase is not complete yet does lane 0 run the bounded wait and the
-// warp follow it.  Every lane sees the same outcome, so the warp-collective
-// tcgen05 instructions after it stay convergent.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort, unsigned* status) {
-  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
-  int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, status) ? 1 : 0;
-  ok = __shfl_sync(0xffffffffu, ok, 0);
-  __syncwarp();
-  return ok != 0;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  uint32_t r;
-  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
-  return r;
-}
-
-// Packed pairs of fp32 (element 0 in the low word) for the f32x2 instructions.
-__device__ __forceinline__ uint64_t f2(float lo, float hi) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-__device__ __forceinline__ void unf2(uint64_t v, float& lo, float& hi) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-}
-__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t r;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
-  return r;
-}
-__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
-  uint64_t r;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-  return r;
-}
-__device__ __forceinline__ float fmax3(float a, float b, float c) {
-  float r;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
-  return r;
-}
-
 // One 32 x 32 fp32 box of this warp's staging (rows of 128 bytes, 16-byte
 // chunk e of row r at chunk e ^ (r & 7): the 128-byte swizzle) to the output
 // at (x, y, z) by a bulk tensor store from lane 0; the staging box stays in
@@ -268,21 +219,10 @@ __device__ __forceinline__ void store_box(const CUtensorMap* map, const unsigned
   }
 }
 
-// A shared-memory descriptor advanced by `bytes`: the start address is the
-// descriptor's low field in 16-byte units, and shared addresses stay below
-// 2^18, so the sum never carries out of it.
-__host__ __device__ constexpr uint64_t desc_step(uint32_t bytes) { return bytes >> 4; }
-
 // Until the bulk store from this warp's staging box has read it.
 __device__ __forceinline__ void staging_free(int lane) {
   if (lane == 0) tc::bulk_wait_read_all();
   __syncwarp();
-}
-
-// Named barrier of the two softmax warps of one TMEM lane quarter (ids 4-7;
-// id 0 is __syncthreads).
-__device__ __forceinline__ void pair_sync(int quarter) {
-  asm volatile("bar.sync %0, 64;" ::"r"(4 + quarter) : "memory");
 }
 
 // Warpgroup register split (setmaxnreg): the two softmax warpgroups take 168

@@ -89,6 +89,9 @@ cudaError_t launch_cross_attn(const AttnArgs& a, cudaStream_t st);
 cudaError_t launch_tree_attn_fma(const AttnArgs& a, cudaStream_t st);
 // Returns cudaErrorNotSupported when the tensor-core kernel does not apply to `a`.
 cudaError_t launch_tree_attn_tc(const AttnArgs& a, cudaStream_t st);
+// Tree verification in 128-row tiles (slabs of more than 64 query rows whose
+// head group divides 128); cudaErrorNotSupported where it does not apply.
+cudaError_t launch_tree_attn_wide(const AttnArgs& a, cudaStream_t st);
 cudaError_t launch_tree_accept(const AcceptArgs& a, cudaStream_t st);
 // Training-time block-mask cross-attention (block_L > 0, T positions per sequence).
 cudaError_t launch_block_attn(const AttnArgs& a, cudaStream_t st);

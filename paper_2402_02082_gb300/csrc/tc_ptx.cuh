@@ -1,6 +1,6 @@
 // Inline-PTX wrappers for the Blackwell (sm_100 family) tensor-core path:
 // tensor memory (TMEM) allocation, tcgen05.mma with shared-memory operand
-// descriptors, tcgen05 loads/stores, and 2-D TMA tensor loads.
+// descriptors, tcgen05 loads/stores, and 2-D / 3-D TMA tensor copies.
 #pragma once
 
 #include <cuda.h>
@@ -156,6 +156,17 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
+// Box of a 3-D tensor map at element coordinates (x, y, z) into shared
+// memory, completing its bytes on `bar`.
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z, uint64_t* bar,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
 }
 

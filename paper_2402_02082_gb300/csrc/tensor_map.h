@@ -1,4 +1,4 @@
-// Host-side helpers for 2-D TMA tensor maps and the launch's shared-memory
+// Host-side helpers for 2-D and 3-D TMA tensor maps and the launch's shared-memory
 // budget, shared by the tensor-core kernels.
 #pragma once
 
@@ -38,6 +38,23 @@ inline bool make_bf16_map(CUtensorMap* m, const void* base, long long rows, long
   const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
   const cuuint32_t es[2] = {1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// A [d2, d1, d0] bf16 tensor (d0 contiguous elements per row) read in boxes
+// of 64 x box1 x box2 elements (64 along d0: 128 bytes, one swizzle atom)
+// with the 128-byte swizzle: the box lands as box1 * box2 rows of 128 bytes,
+// row (z, y) at z * box1 + y.  Out-of-range elements read as zeros.
+inline bool make_bf16_rows3_map(CUtensorMap* m, const void* base, long long d0, long long d1, long long d2, int box1,
+                                int box2) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+  if (!fn) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)d0, (cuuint64_t)d1, (cuuint64_t)d2};
+  const cuuint64_t strides[2] = {(cuuint64_t)d0 * 2, (cuuint64_t)(d0 * d1) * 2};
+  const cuuint32_t box[3] = {64, (cuuint32_t)box1, (cuuint32_t)box2};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }

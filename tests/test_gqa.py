@@ -16,6 +16,8 @@ from gpu_util import assert_attn_close, dev, sample_pairs
 
 pytestmark = pytest.mark.gpu
 
+T64 = gb.GLIDE_FLAG_TILE64
+
 
 @pytest.fixture(scope="module", autouse=True)
 def _lib():
@@ -80,13 +82,25 @@ def test_gqa_cross_attn(B, H, H_kv, D, kv_len, dtype, flags, max_ctas):
     (3, 32, 8, 128, [2000, 33, 900], 6, "random", "bf16", 0, 5),
     (3, 8, 4, 64, [0, 129, 64], 9, "random", "f32", 0, 1000),
     # CaPE-sized trees (33 nodes: 32 verified tokens plus the root) on
-    # Mistral-7B's heads: 132 query rows per cached head, three row tiles
+    # Mistral-7B's heads: 132 query rows per cached head, two row tiles of 128
+    # (three of 64 with GLIDE_FLAG_TILE64)
     (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", 0, 0),
     (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", 0, 5),
+    (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", T64, 0),
+    (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", T64, 5),
     (2, 32, 8, 128, [3000, 200], 33, "random", "bf16", gb.GLIDE_FLAG_FORCE_FMA, 0),
+    (3, 32, 8, 128, [0, 100, 1000], 33, "random", "bf16", 0, 0),   # no prefix; tree keys across a tile edge
+    (3, 32, 8, 128, [0, 100, 1000], 33, "random", "bf16", 0, 7),
+    (2, 32, 8, 128, [257, 2048], 33, "chain", "bf16", 0, 3),
     (1, 32, 8, 128, [1500], 64, "random", "bf16", 0, 0),       # 256 rows: the limit
     (1, 32, 8, 128, [1500], 64, "random", "bf16", 0, 1000),
+    (1, 32, 8, 128, [1500], 64, "random", "bf16", T64, 1000),
+    (2, 16, 8, 128, [900, 40], 40, "random", "bf16", 0, 0),    # group 2: 80 rows, one row tile of 128
+    (2, 64, 8, 128, [600, 1300], 20, "random", "bf16", 0, 9),  # group 8: 160 rows
+    (1, 32, 2, 128, [1100], 10, "random", "bf16", 0, 0),       # group 16: 160 rows
+    (2, 24, 8, 128, [800, 300], 30, "random", "bf16", 0, 4),   # group 3 does not divide 128: 64-row tiles
     (2, 16, 4, 64, [700, 65], 20, "random", "bf16", 0, 7),     # 80 rows, D = 64
+    (2, 16, 4, 64, [700, 65], 20, "random", "bf16", T64, 7),
     (2, 16, 4, 64, [700, 0], 20, "random", "f32", 0, 3),
 ])
 def test_gqa_tree_verify(B, H, H_kv, D, kv_len, n, tree, dtype, flags, max_ctas):
@@ -143,3 +157,21 @@ def test_gqa_bench_shape_sampled():
                       "GQA cross-attention at the bench shape")
     assert_attn_close(ot.cpu().numpy(), oracle.tree_verify_attn(qt, parent, K, V, [L] * B, pairs=pairs), pairs,
                       "GQA verification at the bench shape")
+
+
+def test_gqa_cape_tree_bench_shape_sampled():
+    """Verification of a 33-node CaPE tree on the bench's Mistral-7B shape at
+    full size (B = 4, 32 query over 8 cached heads, D = 128, kv_len 16384:
+    132 query rows per cached head, two row tiles of 128), in the bench's
+    launch configuration, compared with the oracle on sampled (sequence,
+    query head) pairs."""
+    B, H, H_kv, D, L, n = 4, 32, 8, 128, 16384, 33
+    K, V, _, qt, parent = make(B, H, H_kv, D, [L] * B, n, "bf16", seed=4545)
+    S_cap = K.shape[2]
+    ws = ws_for(B, H, H_kv, D, S_cap, n, "bf16")
+    ot = torch.full((B, n, H, D), float("nan"), device="cuda")
+    gb.tree_verify_attn(dev(qt), dev(parent), dev(K), dev(V), dev(np.full(B, L, np.int32)), L, ot, ws)
+    torch.cuda.synchronize()
+    pairs = sample_pairs(B, H, 6, seed=9)
+    assert_attn_close(ot.cpu().numpy(), oracle.tree_verify_attn(qt, parent, K, V, [L] * B, pairs=pairs), pairs,
+                      "GQA 33-node verification at the bench shape")
