@@ -93,8 +93,9 @@ typedef enum { GLIDE_BF16 = 0, GLIDE_F32 = 1 } glide_dtype;
 /* flags */
 #define GLIDE_FLAG_FORCE_FMA 1u   /* tree_verify_attn: use the CUDA-core kernel even where the
                                      tensor-core kernel applies (testing and comparison)     */
-#define GLIDE_FLAG_TILE64 2u      /* tree_verify_attn: serve slabs of more than 64 query rows in
-                                     row tiles of 64 rather than 128 (testing and comparison) */
+#define GLIDE_FLAG_TILE64 2u      /* grouped-query slabs and slabs of more than 64 query rows:
+                                     use the 64-row tensor-core kernel rather than the 128-row
+                                     one (testing and comparison)                            */
 
 typedef struct {
   int32_t B;          /* sequences in the batch, 1..1024                                   */
@@ -109,8 +110,8 @@ typedef struct {
                          H / H_kv consecutive query heads shares one cached head (grouped-
                          query attention, as in Mistral-7B: 32 query over 8 cached heads).
                          tree_verify_attn needs n * H / H_kv <= 256 (query rows per
-                         cached head; more than 64 are served in row tiles of 128 when
-                         H / H_kv divides 128 and the dtype is bf16, else of 64).         */
+                         cached head; with bf16 and H / H_kv dividing 128, grouped-query
+                         slabs are served in row tiles of 128, else in tiles of 64).      */
 } glide_attn_desc;
 
 /* Version of this ABI (GLIDE_ABI_VERSION of the built library). */

@@ -131,6 +131,10 @@ glide_status glide_cross_attn(const glide_attn_desc* desc, const void* q_draft, 
   // kernels without tree keys, with the group's queries as their rows.
   if (a.H / a.Hkv > glide::kMaxRows) return GLIDE_ERR_UNSUPPORTED;
   if (!(a.flags & GLIDE_FLAG_FORCE_FMA)) {
+    if (!(a.flags & GLIDE_FLAG_TILE64)) {
+      cudaError_t e = glide::launch_tree_attn_wide(a, st);
+      if (e != cudaErrorNotSupported) return from_cuda(e);
+    }
     cudaError_t e = glide::launch_tree_attn_tc(a, st);
     if (e != cudaErrorNotSupported) return from_cuda(e);
   }
@@ -153,7 +157,7 @@ glide_status tree_verify_attn(const glide_attn_desc* desc, const void* q_tree, i
   glide::AttnArgs a = make_args(desc, q_tree, K_cache, V_cache, kv_len, parent_idx, out, workspace, n, max_kv_len);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (!(a.flags & GLIDE_FLAG_FORCE_FMA)) {
-    if (!(a.flags & GLIDE_FLAG_TILE64)) {  // slabs of more than 64 query rows: 128-row tiles
+    if (!(a.flags & GLIDE_FLAG_TILE64)) {  // grouped-query slabs and slabs of more than 64 rows: 128-row tiles
       cudaError_t e = glide::launch_tree_attn_wide(a, st);
       if (e != cudaErrorNotSupported) return from_cuda(e);
     }

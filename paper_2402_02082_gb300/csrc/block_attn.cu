@@ -90,9 +90,16 @@ constexpr uint32_t kTmemO = kSBufs * kBN;   // the O accumulator from column 384
 constexpr uint32_t kAtom = 128 * 128;       // one 128-byte-swizzle atom of 128 rows
 constexpr float kRescaleLog2 = 8.0f;
 
+// ODONE has four slots (tile mod 4).  P.V completions are waited on only now
+// and then (a rescale, the epilogue), when up to three products may still be
+// in flight: P.V of tile i - 3 has completed once S of tile i has been read,
+// but those of tiles i - 2 .. i may not have.  Four slots keep every such wait
+// within one phase of its barrier; with two, a wait for tile i could pass on
+// the completion of tile i - 2 (measured: the last tiles of a segment missing
+// from O when the values arrived late from DRAM).
 constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
-              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_OFREE = 29, B_MDONE = 30, B_LREADY = 32, B_LFREE = 33,
-              kNumBars = 34;
+              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_OFREE = 31, B_MDONE = 32, B_LREADY = 34, B_LFREE = 35,
+              kNumBars = 36;
 
 template <int D>
 struct BlkCfg {
@@ -433,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int ks = 1; ks < kBN / 16; ++ks)
               tc::mma_bf16_ts(tmem + kTmemO, pcol + (ks >> 2) * 64 + (ks & 3) * 8, dV + desc_step(ks * 16 * 128), idO, 1u);
             tc::mma_commit(&bars[B_VEMPTY + i % v_stages]);
-            tc::mma_commit(&bars[B_ODONE + (i & 1)]);
+            tc::mma_commit(&bars[B_ODONE + (i & 3)]);
             tc::mma_commit(&bars[B_BFREE + bi]);
           }
         }
@@ -479,7 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&bars[B_LFREE]);
       ++ke;
       const float inv = has_value ? 1.f / (l0 + l1) : 0.f;
-      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 3)], (jl >> 2) & 1, abort_flag, p.status);
       // rounds of two chunks: read from TMEM into the two boxes, then their stores
 #pragma unroll 1
       for (int c2 = 0; c2 < D / 32; c2 += 2) {
@@ -584,7 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float f = need ? fast_exp2(m_used - m_new) : 1.f;
           l *= f;
           if (t > 0 && !dead) {  // O holds the P.V of this item's earlier tiles: rescale this group's half
-            dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 1)], ((i - 1) >> 1) & 1, abort_flag, p.status);
+            dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 3)], ((i - 1) >> 2) & 1, abort_flag, p.status);
             if (!dead) {
               tc::fence_after_sync();
 #pragma unroll 1

@@ -1,7 +1,10 @@
 // Tree verification attention in 128-row tiles on the tcgen05 tensor cores,
-// for grouped-query slabs with more than 64 query rows (Section 3.2's
-// verification of a CaPE tree, under the ancestor-or-self mask, on a target
-// with fewer cached heads than query heads such as Mistral-7B, Section 4.1).
+// for grouped-query slabs (Section 3.2's verification of a CaPE tree, under
+// the ancestor-or-self mask, on a target with fewer cached heads than query
+// heads such as Mistral-7B, Section 4.1) and any slab of more than 64 query
+// rows; without tree keys (a prefix-only mode) the same kernel serves the
+// draft's grouped-query cross-attention (Section 3.1), the group's queries as
+// a slab's rows.
 //
 // A slab is a (sequence, cached head) with n tree nodes x H / H_kv query
 // heads as its rows, node-major: a 33-node CaPE tree on Mistral-7B's 32 query
@@ -49,7 +52,8 @@
 // ancestor-or-self of i (the set built from the parent array by pointer
 // jumping, at the first tile that reaches the tree keys); keys past the
 // prefix and the n tree keys are masked, and their V rows are zeroed in
-// shared memory before P.V (the cache beyond them may hold anything).
+// shared memory before P.V (the cache beyond them may hold anything).  In the
+// prefix-only mode a sequence without cached keys gets zeros.
 // Online softmax in the log2 domain with a lazy reference max: O is rescaled
 // in TMEM only when a tile's max exceeds the reference by more than 8.
 #include <cuda.h>
@@ -83,8 +87,15 @@ constexpr float kRescaleLog2 = 8.0f;
 // segment's epilogue and the pipeline start of the next, with its queries).
 constexpr int kSegWeight = 4;
 
+// ODONE has four slots (tile mod 4).  P.V completions are waited on only now
+// and then (a rescale, the epilogue), when up to three products may still be
+// in flight: P.V of tile i - 3 has completed once S of tile i has been read,
+// but those of tiles i - 2 .. i may not have.  Four slots keep every such wait
+// within one phase of its barrier; with two, a wait for tile i could pass on
+// the completion of tile i - 2 (measured: the last tiles of a segment missing
+// from O when the values arrived late from DRAM).
 constexpr int B_KFULL = 0, B_KEMPTY = 4, B_VFULL = 8, B_VEMPTY = 12, B_QFULL = 16, B_QEMPTY = 17, B_SFULL = 18,
-              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_MDONE = 29, kNumBars = 31;
+              B_PFULL = 21, B_BFREE = 24, B_ODONE = 27, B_MDONE = 31, kNumBars = 33;
 
 template <int D>
 struct WideCfg {
@@ -117,6 +128,7 @@ struct WideParams {
   int B, H, Hkv, group, S_cap, max_kv_len, n;
   int rows;          // query rows per slab: n nodes x group heads, node-major
   int R;             // row tiles of 128 per slab
+  int tree;          // 1: the n tree keys follow the prefix (verification); 0: prefix only
   int nk, nv;        // K and V ring stages
   float scale_log2;
 };
@@ -158,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tmem_relinquish();
   }
   tc::fence_before_sync();
-  build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.n, kBN);  // __syncthreads inside
+  build_batch_tiles(bt, p.kv_len, p.B, p.Hkv, p.max_kv_len, p.tree ? p.n : 0, kBN);  // __syncthreads inside
   tc::fence_after_sync();
   const uint32_t tmem = *tmem_slot;
 
@@ -313,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               tc::mma_bf16_ts(tmem + kTmemO, pcol + (ks >> 2) * 64 + (ks & 3) * 8, dV + desc_step(ks * 16 * 128),
                               idO, 1u);
             tc::mma_commit(&bars[B_VEMPTY + i % nv]);
-            tc::mma_commit(&bars[B_ODONE + (i & 1)]);
+            tc::mma_commit(&bars[B_ODONE + (i & 3)]);
             tc::mma_commit(&bars[B_BFREE + bi]);
           }
         }
@@ -351,6 +363,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         p.ranges[bh] = rg;
       }
+    if (!p.tree) {  // prefix only: a sequence without cached keys gets zeros (an empty softmax)
+      const long long total = (long long)p.B * p.n * p.H * D;
+      for (long long idx = (long long)blockIdx.x * kST + sid; idx < total; idx += (long long)gridDim.x * kST)
+        if (bt.ntiles[idx / ((long long)p.n * p.H * D)] == 0) p.out[idx] = 0.f;
+    }
 
     int i = 0;  // CTA-local key tile
     for (long long g = g_begin; g < g_end;) {
@@ -378,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // the rows of c's descendants-or-self, and nothing past the tree
         const int k0 = t * kBN + kh * 64;
         if (k0 + 64 > plen) {  // warp-uniform
-          if (!anc_ready) {
+          if (p.tree && !anc_ready) {
             anc = ancestors(p.parent + (size_t)s.b * p.n, p.n, node, valid, lane);
             anc_ready = true;
           }
@@ -421,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float f = need ? fast_exp2(m_used - m_new) : 1.f;
           l *= f;
           if (t > s.t0 && !dead) {  // O holds the P.V of this segment's earlier tiles: rescale this group's half
-            dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 1)], ((i - 1) >> 1) & 1, abort_flag, p.status);
+            dead = !warp_wait(&bars[B_ODONE + ((i - 1) & 3)], ((i - 1) >> 2) & 1, abort_flag, p.status);
             if (!dead) {
               tc::fence_after_sync();
 #pragma unroll 1
@@ -485,7 +502,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       pair_sync(quarter);
       const float L = lsum[r] + lsum[kBM + r];
       const int jl = i - 1;  // the segment's last tile
-      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 1)], (jl >> 1) & 1, abort_flag, p.status);
+      if (!dead) dead = !warp_wait(&bars[B_ODONE + (jl & 3)], (jl >> 2) & 1, abort_flag, p.status);
       if (!dead) {
         tc::fence_after_sync();
         uint32_t o[D / 2];
@@ -564,11 +581,12 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
   p.max_kv_len = a.max_kv_len; p.n = a.nq;
   p.rows = a.nq * group;
   p.R = (p.rows + kBM - 1) / kBM;
+  p.tree = a.tree;
   p.nk = nk;
   p.nv = nv;
   p.scale_log2 = a.scale * kLog2e;
   // G shares of the key tiles, R CTAs (row tiles) per share
-  const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + a.nq + kBN - 1) / kBN);
+  const long long tiles_ub = (long long)a.B * a.Hkv * ((a.max_kv_len + (a.tree ? a.nq : 0) + kBN - 1) / kBN);
   long long G = a.max_ctas > 0 ? a.max_ctas : sm_count() / p.R;
   if (G > kMaxCtas) G = kMaxCtas;
   if (G > tiles_ub) G = tiles_ub;
@@ -582,9 +600,11 @@ cudaError_t launch_typed(const AttnArgs& a, cudaStream_t st) {
 }  // namespace
 
 cudaError_t launch_tree_attn_wide(const AttnArgs& a, cudaStream_t st) {
-  if (a.dtype != 0 || (a.D != 128 && a.D != 64) || !a.tree || a.Hkv < 1) return cudaErrorNotSupported;
+  if (a.dtype != 0 || (a.D != 128 && a.D != 64) || a.Hkv < 1) return cudaErrorNotSupported;
   const int group = a.H / a.Hkv;
-  if (a.nq * group <= 64 || a.nq * group > kMaxRows || kBM % group != 0) return cudaErrorNotSupported;
+  // Grouped-query slabs, and any slab of more than 64 rows; multi-head slabs
+  // of up to 64 rows stream faster through the 64-row kernel's deeper rings.
+  if ((group == 1 && a.nq <= 64) || a.nq * group > kMaxRows || kBM % group != 0) return cudaErrorNotSupported;
   // 32-bit TMA coordinates, including a tile's reach past the last row
   if ((long long)a.B * a.Hkv * a.S_cap + kBN > 0x7fffffffLL || (long long)a.B * a.nq + kBM > 0x7fffffffLL)
     return cudaErrorNotSupported;

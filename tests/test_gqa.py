@@ -12,7 +12,7 @@ import oracle
 from paper_2402_02082_gb300 import binding as gb
 from paper_2402_02082_gb300 import build, synth
 
-from gpu_util import assert_attn_close, dev, sample_pairs
+from gpu_util import assert_attn_close, dev
 
 pytestmark = pytest.mark.gpu
 
@@ -55,6 +55,12 @@ def ws_for(B, H, H_kv, D, S_cap, n, dtype):
     (4, 32, 8, 128, [4096, 100, 2000, 16], "bf16", 0, 3),     # few CTAs: split (b, h), merged
     (4, 32, 8, 128, [4096, 100, 2000, 16], "bf16", 0, 1000),
     (2, 16, 4, 128, [300, 700], "f32", 0, 7),
+    # the same cases on the 64-row kernel (GLIDE_FLAG_TILE64), and a group of 3,
+    # which does not divide 128
+    (2, 32, 8, 128, [1000, 37], "bf16", T64, 0),
+    (3, 8, 2, 64, [0, 513, 64], "bf16", T64, 0),
+    (4, 32, 8, 128, [4096, 100, 2000, 16], "bf16", T64, 3),
+    (2, 24, 8, 128, [700, 50], "bf16", 0, 0),
 ])
 def test_gqa_cross_attn(B, H, H_kv, D, kv_len, dtype, flags, max_ctas):
     K, V, qd, _, _ = make(B, H, H_kv, D, kv_len, 1, dtype, seed=700 + H + D)
@@ -75,6 +81,7 @@ def test_gqa_cross_attn(B, H, H_kv, D, kv_len, dtype, flags, max_ctas):
 
 @pytest.mark.parametrize("B,H,H_kv,D,kv_len,n,tree,dtype,flags,max_ctas", [
     (2, 32, 8, 128, [4096, 300], 6, "chain", "bf16", 0, 0),   # GliDe on Mistral-7B: gamma = 5 chain
+    (2, 32, 8, 128, [4096, 300], 6, "chain", "bf16", T64, 0),
     (2, 32, 8, 128, [4096, 300], 6, "chain", "f32", 0, 0),
     (2, 8, 4, 128, [1500, 64], 26, "random", "bf16", 0, 0),   # 52 query rows per slab
     (1, 16, 4, 64, [777], 16, "random", "bf16", 0, 0),        # 64 rows: a full MMA
@@ -137,41 +144,45 @@ def test_gqa_equal_heads_is_multi_head():
     assert np.array_equal(outs[0], outs[1])
 
 
-def test_gqa_bench_shape_sampled():
+def test_gqa_bench_shape_every_output():
     """Grouped-query attention on the bench's Mistral-7B shape at full size
     (B = 4, 32 query heads over 8 cached heads, D = 128, kv_len 16384, the
-    6-node chain of GliDe with gamma = 5), both calls, compared with the
-    oracle on sampled (sequence, query head) pairs."""
+    6-node chain of GliDe with gamma = 5), both calls in the bench's launch
+    configuration, every output compared with the oracle.  Each call runs
+    three times on both tensor-core kernels: a race in the pipeline (the
+    values arriving late from DRAM) shows as a changed result in some run."""
     B, H, H_kv, D, L, n = 4, 32, 8, 128, 16384, 6
     K, V, qd, qt, parent = make(B, H, H_kv, D, [L] * B, n, "bf16", seed=4343, tree="chain")
     S_cap = K.shape[2]
     ws = ws_for(B, H, H_kv, D, S_cap, n, "bf16")
     Kd, Vd, kv = dev(K), dev(V), dev(np.full(B, L, np.int32))
-    oc = torch.full((B, 1, H, D), float("nan"), device="cuda")
-    ot = torch.full((B, n, H, D), float("nan"), device="cuda")
-    gb.glide_cross_attn(dev(qd), Kd, Vd, kv, L, oc, ws)
-    gb.tree_verify_attn(dev(qt), dev(parent), Kd, Vd, kv, L, ot, ws)
-    torch.cuda.synchronize()
-    pairs = sample_pairs(B, H, 6, seed=8)
-    assert_attn_close(oc.cpu().numpy(), oracle.cross_attn(qd, K, V, [L] * B, pairs=pairs), pairs,
-                      "GQA cross-attention at the bench shape")
-    assert_attn_close(ot.cpu().numpy(), oracle.tree_verify_attn(qt, parent, K, V, [L] * B, pairs=pairs), pairs,
-                      "GQA verification at the bench shape")
+    want_c = oracle.cross_attn(qd, K, V, [L] * B)
+    want_t = oracle.tree_verify_attn(qt, parent, K, V, [L] * B)
+    qdd, qtd, pd = dev(qd), dev(qt), dev(parent)
+    for flags in (0, T64):
+        for rep in range(3):
+            oc = torch.full((B, 1, H, D), float("nan"), device="cuda")
+            ot = torch.full((B, n, H, D), float("nan"), device="cuda")
+            gb.glide_cross_attn(qdd, Kd, Vd, kv, L, oc, ws, flags=flags)
+            gb.tree_verify_attn(qtd, pd, Kd, Vd, kv, L, ot, ws, flags=flags)
+            torch.cuda.synchronize()
+            assert_attn_close(oc.cpu().numpy(), want_c, None, f"GQA cross-attention, bench shape, flags {flags}, run {rep}")
+            assert_attn_close(ot.cpu().numpy(), want_t, None, f"GQA verification, bench shape, flags {flags}, run {rep}")
 
 
-def test_gqa_cape_tree_bench_shape_sampled():
+def test_gqa_cape_tree_bench_shape_every_output():
     """Verification of a 33-node CaPE tree on the bench's Mistral-7B shape at
     full size (B = 4, 32 query over 8 cached heads, D = 128, kv_len 16384:
     132 query rows per cached head, two row tiles of 128), in the bench's
-    launch configuration, compared with the oracle on sampled (sequence,
-    query head) pairs."""
+    launch configuration, every output compared with the oracle, three runs."""
     B, H, H_kv, D, L, n = 4, 32, 8, 128, 16384, 33
     K, V, _, qt, parent = make(B, H, H_kv, D, [L] * B, n, "bf16", seed=4545)
     S_cap = K.shape[2]
     ws = ws_for(B, H, H_kv, D, S_cap, n, "bf16")
-    ot = torch.full((B, n, H, D), float("nan"), device="cuda")
-    gb.tree_verify_attn(dev(qt), dev(parent), dev(K), dev(V), dev(np.full(B, L, np.int32)), L, ot, ws)
-    torch.cuda.synchronize()
-    pairs = sample_pairs(B, H, 6, seed=9)
-    assert_attn_close(ot.cpu().numpy(), oracle.tree_verify_attn(qt, parent, K, V, [L] * B, pairs=pairs), pairs,
-                      "GQA 33-node verification at the bench shape")
+    want = oracle.tree_verify_attn(qt, parent, K, V, [L] * B)
+    args = (dev(qt), dev(parent), dev(K), dev(V), dev(np.full(B, L, np.int32)), L)
+    for rep in range(3):
+        ot = torch.full((B, n, H, D), float("nan"), device="cuda")
+        gb.tree_verify_attn(*args, ot, ws)
+        torch.cuda.synchronize()
+        assert_attn_close(ot.cpu().numpy(), want, None, f"GQA 33-node verification at the bench shape, run {rep}")
