@@ -186,3 +186,32 @@ def test_gqa_cape_tree_bench_shape_every_output():
         gb.tree_verify_attn(*args, ot, ws)
         torch.cuda.synchronize()
         assert_attn_close(ot.cpu().numpy(), want, None, f"GQA 33-node verification at the bench shape, run {rep}")
+
+
+def test_gqa_many_sequences_on_128_row_tiles():
+    """Three hundred sequences of short, ragged contexts (some empty) on the
+    128-row kernel: a partition over 600 slabs, a batch table large enough
+    that the launch takes fewer value stages, two row tiles per slab for the
+    33-node trees, and the prefix-only mode with its zero rows, all against
+    the oracle."""
+    B, H, H_kv, D, n = 300, 8, 2, 128, 33
+    kv_len = [int(x) for x in np.random.default_rng(5).integers(0, 260, B)]
+    kv_len[0] = 0
+    kv_len[7] = 0
+    K, V, qd, qt, parent = make(B, H, H_kv, D, kv_len, n, "bf16", seed=951)
+    S_cap = K.shape[2]
+    ws = ws_for(B, H, H_kv, D, S_cap, n, "bf16")
+    Kd, Vd, kv = dev(K), dev(V), dev(np.asarray(kv_len, np.int32))
+    oc = torch.full((B, 1, H, D), float("nan"), device="cuda")
+    ot = torch.full((B, n, H, D), float("nan"), device="cuda")
+    gb.glide_cross_attn(dev(qd), Kd, Vd, kv, max(kv_len), oc, ws)
+    gb.tree_verify_attn(dev(qt), dev(parent), Kd, Vd, kv, max(kv_len), ot, ws)
+    torch.cuda.synchronize()
+    want_c = oracle.cross_attn(qd, K, V, kv_len)
+    for b, L in enumerate(kv_len):
+        if L == 0:
+            assert np.all(oc[b].cpu().numpy() == 0.0), "an empty sequence must give zeros"
+            want_c[b] = 0.0
+    assert_attn_close(oc.cpu().numpy(), want_c, None, "GQA cross, 300 ragged sequences")
+    assert_attn_close(ot.cpu().numpy(), oracle.tree_verify_attn(qt, parent, K, V, kv_len), None,
+                      "GQA verification, 300 ragged sequences")
