@@ -18,8 +18,9 @@
 // which does four times the (row, key) pairs of a 64 x 64 tile per softmax
 // pass; at one row tile that leaves the loop ~20% faster than the HBM pace of
 // an SM, where the 64-row kernel's loop runs right at it, so grouped-query
-// slabs of few rows come here too.  Tensor memory holds three S buffers of 128 columns (S of tile i + 3
-// waits for P.V of tile i) and the O accumulator.  Two softmax groups of four
+// slabs of few rows come here too.  Tensor memory holds three S buffers of
+// 128 columns (S of tile i + 3 waits for P.V of tile i) and the O
+// accumulator.  Two softmax groups of four
 // warps take the two 64-key halves of every tile, one thread per row; the two
 // threads of a row agree on each tile's row max through one TMEM column, so
 // both halves use one reference max and accumulate into the one O, and each
